@@ -1,0 +1,153 @@
+"""Python front end of the fp64 CPU oracle (wise_oracle.c).
+
+TEST INFRASTRUCTURE ONLY: the tests, the smoke check and the benchmark's CPU
+baseline may use this module; the library never imports it.  It compiles the
+C oracle with the host gcc (OpenMP) into oracle/_build/ and calls it through
+ctypes.  Each function states the equation of the paper it evaluates.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "wise_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD, "libwise_oracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+class _Shape(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int), ("seqlen", ctypes.c_int), ("n_heads", ctypes.c_int),
+                ("n_kv_heads", ctypes.c_int), ("head_dim", ctypes.c_int), ("block", ctypes.c_int),
+                ("scale", ctypes.c_double)]
+
+
+class _Select(ctypes.Structure):
+    _fields_ = [("n_sink", ctypes.c_int), ("n_local", ctypes.c_int), ("mode", ctypes.c_int),
+                ("topk", ctypes.c_int), ("eta", ctypes.c_float), ("cap", ctypes.c_int)]
+
+
+def build(force: bool = False) -> str:
+    """Compile the C oracle (gcc -O2 -fopenmp) if it is missing or stale."""
+    with _lock:
+        if force or not os.path.exists(_LIB_PATH) or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC):
+            os.makedirs(_BUILD, exist_ok=True)
+            tmp = _LIB_PATH + f".{os.getpid()}.tmp"
+            subprocess.check_call(["gcc", "-O2", "-fopenmp", "-shared", "-fPIC", "-o", tmp, _SRC, "-lm"])
+            os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        lib = ctypes.CDLL(build())
+        P = ctypes.c_void_p
+        lib.wo_full_attention.argtypes = [ctypes.POINTER(_Shape), P, P, P, ctypes.c_long, P, P, P]
+        lib.wo_sparse_attention.argtypes = [ctypes.POINTER(_Shape), P, P, P, P, P, ctypes.c_int,
+                                            ctypes.c_long, P, P]
+        lib.wo_select_support.argtypes = [ctypes.POINTER(_Shape), ctypes.POINTER(_Select), P, P, P]
+        lib.wo_max_threads.restype = ctypes.c_int
+        lib.wo_set_threads.argtypes = [ctypes.c_int]
+        _lib = lib
+    return _lib
+
+
+def set_threads(n: int) -> None:
+    _load().wo_set_threads(int(n))
+
+
+def max_threads() -> int:
+    return int(_load().wo_max_threads())
+
+
+def _shape(batch, seqlen, n_heads, n_kv_heads, head_dim, block, scale=0.0):
+    return _Shape(batch, seqlen, n_heads, n_kv_heads, head_dim, block, float(scale or 0.0))
+
+
+def _ptr(a):
+    return a.ctypes.data_as(ctypes.c_void_p) if a is not None else None
+
+
+def _bits(a):
+    a = np.ascontiguousarray(a)
+    if a.dtype != np.uint16:
+        raise TypeError("bf16 inputs are passed as uint16 bit patterns")
+    return a
+
+
+def _units(units):
+    if units is None:
+        return None, 0
+    u = np.ascontiguousarray(np.asarray(units, dtype=np.int32).reshape(-1, 3))
+    return u, len(u)
+
+
+def full_attention(Q, K, V, block, units=None, scale=None, with_mass=True):
+    """Eq. 2 (causal mask) and Eq. 5.
+
+    Q [B,H,L,D], K/V [B,Hkv,L,D] as bf16 bits.  Returns (O, mass) in float64:
+    O [B,H,L,D] and mass [B,H,nQB,nKB] for all query blocks, or packed per
+    listed (b, h, q) unit: O [n,block,D], mass [n,nKB].
+    """
+    Q, K, V = _bits(Q), _bits(K), _bits(V)
+    B, H, L, D = Q.shape
+    Hkv = K.shape[1]
+    nb = L // block
+    u, n = _units(units)
+    if u is None:
+        O = np.zeros((B, H, L, D), dtype=np.float64)
+        M = np.zeros((B, H, nb, nb), dtype=np.float64) if with_mass else None
+    else:
+        O = np.zeros((n, block, D), dtype=np.float64)
+        M = np.zeros((n, nb), dtype=np.float64) if with_mass else None
+    sh = _shape(B, L, H, Hkv, D, block, scale)
+    rc = _load().wo_full_attention(ctypes.byref(sh), _ptr(Q), _ptr(K), _ptr(V), n, _ptr(u), _ptr(O), _ptr(M))
+    if rc != 0:
+        raise ValueError("oracle full_attention rejected its arguments")
+    return O, M
+
+
+def sparse_attention(Q, K, V, idx, counts, block, units=None, scale=None):
+    """Eqs. 7-8: attention restricted to the block support (idx, counts)."""
+    Q, K, V = _bits(Q), _bits(K), _bits(V)
+    B, H, L, D = Q.shape
+    Hkv = K.shape[1]
+    idx = np.ascontiguousarray(idx, dtype=np.int32)
+    counts = np.ascontiguousarray(counts, dtype=np.int32)
+    cap = idx.shape[-1]
+    u, n = _units(units)
+    O = np.zeros((B, H, L, D) if u is None else (n, block, D), dtype=np.float64)
+    sh = _shape(B, L, H, Hkv, D, block, scale)
+    rc = _load().wo_sparse_attention(ctypes.byref(sh), _ptr(Q), _ptr(K), _ptr(V), _ptr(idx), _ptr(counts),
+                                     cap, n, _ptr(u), _ptr(O))
+    if rc != 0:
+        raise ValueError("oracle sparse_attention rejected its arguments")
+    return O
+
+
+def select_support(blockmass, n_kv_heads, block, mode, n_sink, n_local, topk, eta, cap):
+    """Eq. 6 in single-pass form: forced sink/local blocks, then top-k or
+    cumulative-mass coverage over the pooled fixed-point masses.
+
+    blockmass [B,H,nQB,nKB] float32.  Returns idx [B,Hkv,nQB,cap] int32
+    (ascending, -1 padded) and counts [B,Hkv,nQB] int32.
+    """
+    m = np.ascontiguousarray(blockmass, dtype=np.float32)
+    B, H, nq, nk = m.shape
+    if nq != nk:
+        raise ValueError("blockmass must be square in its last two dims")
+    idx = np.empty((B, n_kv_heads, nq, cap), dtype=np.int32)
+    counts = np.empty((B, n_kv_heads, nq), dtype=np.int32)
+    sh = _shape(B, nq * block, H, n_kv_heads, 1, block)
+    sel = _Select(int(n_sink), int(n_local), int(mode), int(topk), float(eta), int(cap))
+    rc = _load().wo_select_support(ctypes.byref(sh), ctypes.byref(sel), _ptr(m), _ptr(idx), _ptr(counts))
+    if rc != 0:
+        raise ValueError("oracle select_support rejected its arguments")
+    return idx, counts

@@ -1,0 +1,344 @@
+"""Pins of the fp64 oracle to facts fixed by the paper and by mathematics.
+
+None of these tests compares the oracle with itself.  Each one checks it
+against a library routine (torch's fp64 scaled-dot-product attention and
+softmax), a closed form, an invariant the equations imply, a hand-derived
+case, or an exhaustive search over the definition, chosen so that a dropped
+term, a wrong sign, a swapped index or a transposed operand fails at least
+one of them.
+"""
+import itertools
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as orc
+from paper_2609_27373_gb300 import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def bf16_vals(bits):
+    return synth.bf16_bits_to_f32(bits).astype(np.float64)
+
+
+def expand_kv(x, group):
+    return np.repeat(x, group, axis=1)
+
+
+def sdpa_reference(Q, K, V, group, attn_mask=None, is_causal=False, scale=None):
+    """torch fp64 scaled_dot_product_attention on the widened bf16 values."""
+    q = torch.from_numpy(bf16_vals(Q))
+    k = torch.from_numpy(expand_kv(bf16_vals(K), group))
+    v = torch.from_numpy(expand_kv(bf16_vals(V), group))
+    m = None if attn_mask is None else torch.from_numpy(attn_mask)
+    return torch.nn.functional.scaled_dot_product_attention(q, k, v, attn_mask=m, is_causal=is_causal,
+                                                            scale=scale).numpy()
+
+
+# --------------------------------------------------------------------------- Eq. 2
+
+@pytest.mark.parametrize("B,H,Hkv,L,D,blk", [(2, 4, 2, 48, 8, 16), (1, 3, 3, 40, 5, 8), (1, 2, 1, 12, 3, 4)])
+def test_full_attention_equals_library_causal_sdpa(B, H, Hkv, L, D, blk):
+    """Eq. 2 with a causal M is torch's causal scaled-dot-product attention
+    (scale 1/sqrt(d_h)); GQA heads share their group's K/V."""
+    Q, K, V = synth.random_qkv(B, H, Hkv, L, D, seed=11 + L)
+    O, _ = orc.full_attention(Q, K, V, blk)
+    ref = sdpa_reference(Q, K, V, H // Hkv, is_causal=True)
+    np.testing.assert_allclose(O, ref, rtol=0, atol=1e-12)
+
+
+def test_full_attention_custom_scale():
+    Q, K, V = synth.random_qkv(1, 2, 2, 16, 4, seed=3)
+    O, _ = orc.full_attention(Q, K, V, 4, scale=0.37)
+    ref = sdpa_reference(Q, K, V, 1, is_causal=True, scale=0.37)
+    np.testing.assert_allclose(O, ref, rtol=0, atol=1e-12)
+
+
+def test_one_hot_routing_closed_form():
+    """Query i aims at key j*(i) <= i with logit 16, every other admissible
+    logit is 0: O_i = (e^16 V_j* + sum_{j<=i, j!=j*} V_j) / (e^16 + i)."""
+    L = D = 16
+    rng = np.random.default_rng(5)
+    target = np.array([rng.integers(0, i + 1) for i in range(L)])
+    K = np.zeros((1, 1, L, D), np.float32)
+    Q = np.zeros((1, 1, L, D), np.float32)
+    for j in range(L):
+        K[0, 0, j, j] = 8.0
+    for i in range(L):
+        Q[0, 0, i, target[i]] = 8.0          # logit = (8*8) / sqrt(16) = 16
+    V = rng.standard_normal((1, 1, L, D)).astype(np.float32)
+    Qb, Kb, Vb = (synth.f32_to_bf16_bits(x) for x in (Q, K, V))
+    O, _ = orc.full_attention(Qb, Kb, Vb, 4)
+    v = bf16_vals(Vb)[0, 0]
+    for i in range(L):
+        others = [j for j in range(i + 1) if j != target[i]]
+        want = (math.exp(16.0) * v[target[i]] + v[others].sum(axis=0)) / (math.exp(16.0) + i)
+        np.testing.assert_allclose(O[0, 0, i], want, rtol=0, atol=1e-12)
+
+
+def test_zero_queries_closed_form():
+    """Q = 0 makes every admissible logit equal: A_ij = 1/(i+1) for j <= i, so
+    O_i = mean_{j<=i} V_j and r_qb = (1/B) sum_{i in I_q} |{j in I_b: j<=i}|/(i+1)."""
+    L, D, blk = 24, 6, 4
+    _, K, V = synth.random_qkv(1, 1, 1, L, D, seed=9)
+    Q = np.zeros((1, 1, L, D), np.uint16)
+    O, M = orc.full_attention(Q, K, V, blk)
+    v = bf16_vals(V)[0, 0]
+    want_o = np.cumsum(v, axis=0) / np.arange(1, L + 1)[:, None]
+    np.testing.assert_allclose(O[0, 0], want_o, rtol=0, atol=1e-13)
+    nb = L // blk
+    want_m = np.zeros((nb, nb))
+    for q in range(nb):
+        for b in range(nb):
+            for i in range(q * blk, (q + 1) * blk):
+                n_keys = sum(1 for j in range(b * blk, (b + 1) * blk) if j <= i)
+                want_m[q, b] += n_keys / (i + 1) / blk
+    np.testing.assert_allclose(M[0, 0], want_m, rtol=0, atol=1e-14)
+
+
+# --------------------------------------------------------------------------- Eq. 5
+
+def test_block_mass_equals_library_softmax_block_sums():
+    """Eq. 5 from torch's fp64 softmax of the causally masked logits, summed
+    over key blocks and averaged over the |I_q| = B query rows."""
+    B, H, Hkv, L, D, blk = 1, 4, 2, 32, 8, 8
+    Q, K, V = synth.random_qkv(B, H, Hkv, L, D, seed=21)
+    _, M = orc.full_attention(Q, K, V, blk)
+    q = torch.from_numpy(bf16_vals(Q))
+    k = torch.from_numpy(expand_kv(bf16_vals(K), H // Hkv))
+    logits = q @ k.transpose(-1, -2) / math.sqrt(D)
+    causal = torch.ones(L, L, dtype=torch.bool).tril()
+    A = torch.softmax(logits.masked_fill(~causal, float("-inf")), dim=-1)
+    nb = L // blk
+    want = A.reshape(B, H, nb, blk, nb, blk).sum(dim=(3, 5)) / blk
+    np.testing.assert_allclose(M, want.numpy(), rtol=0, atol=1e-14)
+
+
+def test_block_mass_rows_sum_to_one_and_are_causal():
+    """Rows of A sum to 1 (Eq. 2), hence sum_b r_qb = 1 (Eq. 5); r_qb = 0 for b > q."""
+    Q, K, V = synth.random_qkv(2, 3, 3, 64, 16, seed=4, std=2.0)
+    _, M = orc.full_attention(Q, K, V, 16)
+    np.testing.assert_allclose(M.sum(-1), 1.0, rtol=0, atol=1e-13)
+    assert np.all(np.triu(M, k=1) == 0.0)
+    assert np.all(M >= 0.0)
+
+
+def test_units_pack_the_same_rows():
+    Q, K, V = synth.random_qkv(2, 4, 2, 32, 8, seed=8)
+    O, M = orc.full_attention(Q, K, V, 8)
+    units = [(1, 3, 2), (0, 0, 0), (1, 1, 3)]
+    Ou, Mu = orc.full_attention(Q, K, V, 8, units=units)
+    for n, (b, h, q) in enumerate(units):
+        np.testing.assert_array_equal(Ou[n], O[b, h, q * 8:(q + 1) * 8])
+        np.testing.assert_array_equal(Mu[n], M[b, h, q])
+    idx, counts = synth.random_support(2, 2, 4, 3, seed=1)
+    Os = orc.sparse_attention(Q, K, V, idx, counts, 8)
+    Osu = orc.sparse_attention(Q, K, V, idx, counts, 8, units=units)
+    for n, (b, h, q) in enumerate(units):
+        np.testing.assert_array_equal(Osu[n], Os[b, h, q * 8:(q + 1) * 8])
+
+
+def test_bad_arguments_are_rejected():
+    Q, K, V = synth.random_qkv(1, 2, 2, 16, 4, seed=0)
+    with pytest.raises(ValueError):
+        orc.full_attention(Q, K, V, 5)                     # L % B != 0
+    with pytest.raises(ValueError):
+        orc.full_attention(Q, K, V, 4, units=[(0, 2, 0)])  # head out of range
+    idx = np.full((1, 2, 4, 2), 7, np.int32)
+    with pytest.raises(ValueError):
+        orc.sparse_attention(Q, K, V, idx, np.ones((1, 2, 4), np.int32), 4)  # block 7 >= nKB
+
+
+# --------------------------------------------------------------------------- Eqs. 7-8
+
+def test_sparse_with_all_blocks_equals_full():
+    """R == 0 when every admissible block is in the support (Eq. 8 -> Eq. 2)."""
+    B, H, Hkv, L, D, blk = 2, 4, 2, 64, 8, 16
+    Q, K, V = synth.random_qkv(B, H, Hkv, L, D, seed=12)
+    idx, counts = synth.all_blocks_support(B, Hkv, L // blk)
+    O_full, _ = orc.full_attention(Q, K, V, blk)
+    O_sp = orc.sparse_attention(Q, K, V, idx, counts, blk)
+    np.testing.assert_allclose(O_sp, O_full, rtol=0, atol=1e-14)
+
+
+def test_sparse_equals_library_masked_sdpa():
+    """Eq. 8 is softmax(QK^T/sqrt(d) + M + R)V: torch SDPA with the boolean
+    mask (j <= i) and (b(j) in B_q(i))."""
+    B, H, Hkv, L, D, blk = 2, 4, 2, 64, 8, 8
+    nb = L // blk
+    Q, K, V = synth.random_qkv(B, H, Hkv, L, D, seed=13)
+    idx, counts = synth.random_support(B, Hkv, nb, 4, seed=2)
+    O = orc.sparse_attention(Q, K, V, idx, counts, blk)
+    grp = H // Hkv
+    mask = np.zeros((B, H, L, L), dtype=bool)
+    for b in range(B):
+        for h in range(H):
+            for q in range(nb):
+                for kb in idx[b, h // grp, q, : counts[b, h // grp, q]]:
+                    mask[b, h, q * blk:(q + 1) * blk, kb * blk:(kb + 1) * blk] = True
+    mask &= np.tril(np.ones((L, L), dtype=bool))
+    ref = sdpa_reference(Q, K, V, grp, attn_mask=mask)
+    np.testing.assert_allclose(O, ref, rtol=0, atol=1e-12)
+
+
+def test_sparse_diagonal_only_is_blockwise_causal_attention():
+    """With B_q = {q} every query block attends causally inside itself only."""
+    L, D, blk = 32, 8, 8
+    nb = L // blk
+    Q, K, V = synth.random_qkv(1, 2, 2, L, D, seed=14)
+    idx = np.arange(nb, dtype=np.int32).reshape(1, 1, nb, 1).repeat(2, axis=1)
+    counts = np.ones((1, 2, nb), np.int32)
+    O = orc.sparse_attention(Q, K, V, idx, counts, blk)
+    q = bf16_vals(Q).reshape(1, 2, nb, blk, D)
+    k = bf16_vals(K).reshape(1, 2, nb, blk, D)
+    v = bf16_vals(V).reshape(1, 2, nb, blk, D)
+    ref = torch.nn.functional.scaled_dot_product_attention(torch.from_numpy(q), torch.from_numpy(k),
+                                                           torch.from_numpy(v), is_causal=True).numpy()
+    np.testing.assert_allclose(O, ref.reshape(1, 2, L, D), rtol=0, atol=1e-12)
+
+
+def test_sparse_empty_support_rows_are_zero():
+    L, D, blk = 32, 4, 8
+    Q, K, V = synth.random_qkv(1, 1, 1, L, D, seed=15)
+    idx = np.full((1, 1, 4, 2), -1, np.int32)
+    counts = np.zeros((1, 1, 4), np.int32)
+    O = orc.sparse_attention(Q, K, V, idx, counts, blk)
+    assert np.all(O == 0.0)
+
+
+# --------------------------------------------------------------------------- Eq. 6
+
+def _run_case(case):
+    nb, q, group = case["nb"], case["q"], case["group"]
+    m = np.zeros((1, group, nb, nb), np.float32)
+    for h, row in enumerate(case["masses"]):
+        m[0, h, q] = [float("nan") if x == "nan" else x for x in row]
+    mode = synth.SEL_TOPK if case["mode"] == "topk" else synth.SEL_COVERAGE
+    idx, counts = orc.select_support(m, 1, 1, mode, case["n_sink"], case["n_local"], case["topk"],
+                                     case["eta"], case["cap"])
+    return idx[0, 0, q], counts[0, 0, q]
+
+
+with open(os.path.join(GOLDEN, "selection_cases.json")) as _f:
+    _CASES = json.load(_f)["cases"]
+
+
+@pytest.mark.parametrize("case", _CASES, ids=[c["name"] for c in _CASES])
+def test_selection_golden_cases(case):
+    row, n = _run_case(case)
+    assert n == len(case["expect"]), case["why"]
+    assert row[:n].tolist() == case["expect"], case["why"]
+    assert np.all(row[n:] == -1)
+
+
+def _u(x):
+    x = np.float32(x)
+    if not (x > 0):
+        return 0
+    return int(math.floor(float(min(x, np.float32(4096.0))) * 2.0 ** 32))
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_coverage_is_minimum_cardinality_by_exhaustive_search(seed):
+    """Eq. 6 defines B_q as argmin |B| s.t. sum_{b in B} r_qb >= eta.  Search
+    every superset of the forced blocks: the selected set must reach the
+    threshold, have the minimum size, and carry the maximum mass among sets
+    of that size."""
+    rng = np.random.default_rng(seed)
+    nb = 9
+    q = nb - 1
+    group = 1 + seed % 2
+    m = np.zeros((1, group, nb, nb), np.float32)
+    m[0, :, q] = rng.dirichlet(np.full(nb, 0.4), size=group).astype(np.float32)
+    eta = float(rng.choice([0.5, 0.8, 0.9, 0.95]))
+    n_sink, n_local = 1, 1 + seed % 2
+    idx, counts = orc.select_support(m, 1, 1, synth.SEL_COVERAGE, n_sink, n_local, 0, eta, nb)
+    got = set(idx[0, 0, q, : counts[0, 0, q]].tolist())
+    U = [sum(_u(m[0, h, q, kb]) for h in range(group)) for kb in range(nb)]
+    T = sum(U)
+    e16 = int(math.floor(eta * 65536 + 0.5))
+    forced = set(range(n_sink)) | set(range(q - n_local + 1, q + 1))
+    cands = [kb for kb in range(nb) if kb not in forced]
+
+    def ok(S):
+        return sum(U[kb] for kb in S) * 65536 >= e16 * T
+
+    best = None
+    for r in range(len(cands) + 1):
+        sets = [forced | set(c) for c in itertools.combinations(cands, r)]
+        good = [S for S in sets if ok(S)]
+        if good:
+            best = (r, max(sum(U[kb] for kb in S) for S in good))
+            break
+    assert ok(got)
+    assert len(got) == len(forced) + best[0]
+    assert sum(U[kb] for kb in got) == best[1]
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_topk_matches_library_stable_ranking(seed):
+    """Top-k keeps the k best candidates under (pooled mass desc, index asc):
+    numpy's lexsort of the pooled fixed-point masses gives the same set."""
+    rng = np.random.default_rng(100 + seed)
+    B, H, Hkv, nb = 2, 4, 2, 12
+    m = rng.random((B, H, nb, nb)).astype(np.float32)
+    m[..., :, 3] = m[..., :, 4]           # planted exact ties between blocks 3 and 4
+    k, cap, n_sink, n_local = 3, 6, 1, 2
+    idx, counts = orc.select_support(m, Hkv, 1, synth.SEL_TOPK, n_sink, n_local, k, 0.0, cap)
+    grp = H // Hkv
+    for b in range(B):
+        for g in range(Hkv):
+            for q in range(nb):
+                U = np.array([sum(_u(m[b, h, q, kb]) for h in range(g * grp, (g + 1) * grp))
+                              for kb in range(q + 1)], dtype=object)
+                forced = set(range(min(n_sink, q + 1))) | set(range(max(0, q - n_local + 1), q + 1))
+                cands = np.array([kb for kb in range(q + 1) if kb not in forced], dtype=np.int64)
+                if len(cands):
+                    keys = np.array([U[kb] for kb in cands], dtype=np.float64)
+                    order = np.lexsort((cands, -keys))
+                    pick = set(cands[order[: min(k, cap - len(forced))]].tolist())
+                else:
+                    pick = set()
+                want = sorted(forced | pick)
+                assert counts[b, g, q] == len(want)
+                assert idx[b, g, q, : len(want)].tolist() == want
+
+
+def test_selection_rejects_bad_parameters():
+    m = np.zeros((1, 1, 4, 4), np.float32)
+    with pytest.raises(ValueError):
+        orc.select_support(m, 1, 1, synth.SEL_TOPK, 1, 1, 2, 0.0, 1)      # cap < forced
+    with pytest.raises(ValueError):
+        orc.select_support(m, 1, 1, synth.SEL_COVERAGE, 1, 1, 0, 1.5, 4)  # eta > 1
+    with pytest.raises(ValueError):
+        orc.select_support(m, 1, 1, synth.SEL_TOPK, 1, 0, 2, 0.0, 4)      # no diagonal
+
+
+# --------------------------------------------------------------------------- end to end (sanity)
+
+def test_planted_blocks_are_recovered_on_the_tiny_workload():
+    """Statistical sanity of generator + oracle (not a parity check): after
+    the discovery steps, top-k selection recovers the planted key blocks."""
+    wl = synth.WORKLOADS["tiny"]
+    traj = synth.Trajectory(wl)
+    acc = None
+    for t in range(wl.n_discovery):
+        Q, K, V = traj.step(t)
+        _, M = orc.full_attention(Q, K, V, wl.block)
+        acc = M if acc is None else acc + M
+    idx, counts = orc.select_support(acc.astype(np.float32), wl.n_kv_heads, wl.block, wl.sel_mode, wl.n_sink,
+                                     wl.n_local, wl.topk, wl.eta, wl.cap)
+    hit = tot = 0
+    for g in range(wl.n_kv_heads):
+        for q in range(wl.n_blocks):
+            chosen = set(idx[0, g, q, : counts[0, g, q]].tolist())
+            for p in traj.planted[0][g][q]:
+                tot += 1
+                hit += p in chosen
+    assert tot > 0 and hit / tot >= 0.9
+    np.testing.assert_allclose(acc.sum(-1), wl.n_discovery, atol=1e-12)
