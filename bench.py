@@ -1,0 +1,389 @@
+"""Benchmark of the WISE attention hot path on one or more GB300s.
+
+One benchmark step is one recurrent trajectory of the 4K workload (batch 1,
+L=4096, 32 heads, head_dim 128, block 128, T=32): the discovery steps run
+dense attention with the block-mass epilogue, one selection builds the
+support (sink + diagonal + 95% mass coverage, cap 8), and every late step runs
+support-restricted attention.  Every step of the trajectory has its own
+Q/K/V (2.9 GB in total, far above the 129 MB L2), resident in HBM before the
+timed region starts.
+
+Reported (one JSON line on rank 0):
+  value            late-step attention ms per recurrent step (sparse kernel,
+                   CUDA events on the launching stream, mean over late steps)
+  dense_ms         the library's own dense kernel (no mass) on the same late
+                   inputs; speedup = dense_ms / value
+  roofline         the sparse kernel's algorithmic tensor FLOPs per launch
+                   over its mean launch time, against the measured bf16 peak
+  e2e              the same late step through the C ABI with Q/K/V copied from
+                   pinned host memory and O copied back inside the timed region
+  cpu_baseline     the fp64 oracle timed on a bounded sample on the host cores
+Multi-GPU: every rank runs an independent replica (the path has no exchange
+step); value is the max over ranks.
+
+--impl reference times the fp64 oracle (the reference arm of this build) on
+a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+WORKLOAD = "4k"
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    try:
+        with open(PEAKS_FILE) as f:
+            d = json.load(f)
+        return d, "measured"
+    except (OSError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+# --------------------------------------------------------------------------- FLOP accounting
+
+def pair_count(block: int, diagonal: bool) -> int:
+    """Query-key pairs of one (query block, key block) tile: B^2 off the
+    diagonal, B(B+1)/2 on it (causal mask, Eq. 2)."""
+    return block * (block + 1) // 2 if diagonal else block * block
+
+
+def sparse_flops(idx: np.ndarray, counts: np.ndarray, n_heads: int, head_dim: int, block: int) -> float:
+    """4*d FLOPs (QK^T and PV) per computed query-key pair over the support."""
+    B, Hkv, nb, _ = idx.shape
+    group = n_heads // Hkv
+    total = 0
+    for b in range(B):
+        for g in range(Hkv):
+            for q in range(nb):
+                for kb in idx[b, g, q, : counts[b, g, q]]:
+                    total += pair_count(block, kb == q)
+    return 4.0 * head_dim * total * group
+
+
+def dense_flops(batch: int, n_heads: int, seqlen: int, head_dim: int) -> float:
+    return 4.0 * head_dim * batch * n_heads * seqlen * (seqlen + 1) / 2
+
+
+# --------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """Samples SM clocks and throttle reasons with nvidia-smi while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int, path: str):
+        self.path = path
+        self.proc = None
+        try:
+            self.f = open(path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(gpu_index), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"], stdout=self.f,
+                                         stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.close()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# --------------------------------------------------------------------------- oracle (CPU) arm
+
+def oracle_late_step_ms(wl, late_inputs, idx, counts, n_heads_sample: int):
+    """fp64 oracle on `n_heads_sample` heads of one late step, scaled to the
+    full step (work is uniform across heads).  Returns (ms, cores, seconds)."""
+    from oracle import oracle as orc
+    Q, K, V = late_inputs
+    units = [(b, h, q) for b in range(wl.batch) for h in range(n_heads_sample) for q in range(wl.n_blocks)]
+    t0 = time.perf_counter()
+    orc.sparse_attention(Q, K, V, idx, counts, wl.block, units=units)
+    sec = time.perf_counter() - t0
+    scale = (wl.batch * wl.n_heads * wl.n_blocks) / len(units)
+    return 1e3 * sec * scale, orc.max_threads(), sec
+
+
+def run_reference(args):
+    """Reference arm: the fp64 oracle on a bounded sample of the same workload."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    from oracle import oracle as orc
+    from paper_2609_27373_gb300 import synth
+    wl = synth.WORKLOADS[WORKLOAD]
+    traj = synth.Trajectory(wl)
+    acc = None
+    units_all = None
+    # Discovery on the oracle would take minutes at 4K; the support is built
+    # from the oracle's own masses of a 2-head sample and replicated (the
+    # measured quantity is the late step's cost, which depends on the support
+    # sizes only through the cap).
+    sample_heads = 2
+    for t in range(wl.n_discovery):
+        Q, K, V = traj.step(t)
+    Q, K, V = traj.step(wl.n_discovery)
+    units_all = [(0, h, q) for h in range(sample_heads) for q in range(wl.n_blocks)]
+    _, m = orc.full_attention(Q, K, V, wl.block, units=units_all, with_mass=True)
+    mass = np.zeros((wl.batch, wl.n_heads, wl.n_blocks, wl.n_blocks), np.float32)
+    for n, (b, h, q) in enumerate(units_all):
+        mass[b, h::sample_heads, q] = m[n]
+    idx, counts = orc.select_support(mass, wl.n_kv_heads, wl.block, wl.sel_mode, wl.n_sink, wl.n_local, wl.topk,
+                                     wl.eta, wl.cap)
+    times = []
+    for s in range(args.warmup + args.steps):
+        ms, cores, _ = oracle_late_step_ms(wl, (Q, K, V), idx, counts, 1)
+        if s >= args.warmup:
+            times.append(ms)
+    value = statistics.median(times)
+    line = {
+        "impl": "reference", "metric": "late-step attention ms/step (fp64 CPU oracle)", "value": value,
+        "unit": "ms", "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": value, "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f64", "data": "synthetic",
+        "config": {"workload": "4k: batch 1, L=4096, 32 heads, head_dim 128, block 128, T=32, coverage 0.95 cap 8",
+                   "parallelism": "replicas"},
+        "cpu_baseline": {"value": value, "unit": "ms", "cores": cores, "kind": "oracle",
+                         "sample": "1 of 32 heads of one late step per timed step, scaled x32"},
+        "e2e": {"value": value, "unit": "ms", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+# --------------------------------------------------------------------------- GPU arm
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("at least 3 warm-up steps")
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+    import torch.distributed as dist
+    from paper_2609_27373_gb300 import synth, wise
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    wl = synth.WORKLOADS[WORKLOAD]
+    shape, sel = wise.shape_of(wl), wise.select_of(wl)
+    n_late = wl.steps - wl.n_discovery
+
+    # ---- inputs: the whole trajectory, generated on the host, resident in HBM
+    traj = synth.Trajectory(wl)
+    host_steps, dev_steps = [], []
+    for t in range(wl.steps):
+        q, k, v = traj.step(t)
+        host_steps.append((q, k, v))
+        dev_steps.append(tuple(torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).cuda() for x in (q, k, v)))
+    O = torch.empty(host_steps[0][0].shape, dtype=torch.bfloat16, device="cuda")
+    layer = wise.WiseAttention(shape, sel, wl.n_discovery)
+    stream = torch.cuda.current_stream()
+
+    def trajectory(ev=None):
+        layer.selected = False
+        for t in range(wl.steps):
+            Q, K, V = dev_steps[t]
+            if ev is not None:
+                ev[t][0].record(stream)
+            layer.step(t, Q, K, V, O)
+            if ev is not None:
+                ev[t][1].record(stream)
+
+    for _ in range(args.warmup):
+        trajectory()
+    torch.cuda.synchronize()
+    idx_h, counts_h = layer.idx.cpu().numpy(), layer.counts.cpu().numpy()
+    flops_sparse = sparse_flops(idx_h, counts_h, wl.n_heads, wl.head_dim, wl.block)
+    flops_dense = dense_flops(wl.batch, wl.n_heads, wl.seqlen, wl.head_dim)
+    density = flops_sparse / flops_dense
+
+    clocks = ClockSampler(local, os.path.join(ROOT, "gpurun_out" if os.path.isdir(os.path.join(ROOT, "gpurun_out"))
+                                              else ".", f".clocks_rank{rank}.csv"))
+    time.sleep(0.3)
+
+    # ---- timed: K trajectories
+    evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(wl.steps)]
+           for _ in range(args.steps)]
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    torch.cuda.synchronize()
+    t_start.record(stream)
+    for k in range(args.steps):
+        trajectory(evs[k])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    total_ms = t_start.elapsed_time(t_end)
+    disc_ms, sel_ms, late_ms = [], [], []
+    for k in range(args.steps):
+        for t in range(wl.steps):
+            ms = evs[k][t][0].elapsed_time(evs[k][t][1])
+            if t < wl.n_discovery:
+                disc_ms.append(ms)
+            elif t == wl.n_discovery:
+                late_ms.append(ms)  # includes the selection launch; split below
+            else:
+                late_ms.append(ms)
+    # the first late step also ran the selection; time the selection alone
+    sel_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    for k in range(args.steps):
+        sel_ev[k][0].record(stream)
+        wise.wise_select_support(shape, sel, layer.blockmass, layer.idx, layer.counts)
+        sel_ev[k][1].record(stream)
+    torch.cuda.synchronize()
+    sel_ms = [a.elapsed_time(b) for a, b in sel_ev]
+    late_only = [late_ms[i] for i in range(len(late_ms)) if i % n_late != 0]  # steps without the selection
+
+    # ---- own dense kernel on the same late inputs
+    dense_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_late)]
+    dense_ms = []
+    for k in range(max(1, args.steps // 2)):
+        for i, t in enumerate(range(wl.n_discovery, wl.steps)):
+            Q, K, V = dev_steps[t]
+            dense_ev[i][0].record(stream)
+            wise.wise_full_attn_accumulate(shape, Q, K, V, O)
+            dense_ev[i][1].record(stream)
+        torch.cuda.synchronize()
+        dense_ms += [a.elapsed_time(b) for a, b in dense_ev]
+
+    # ---- end to end through host buffers (pinned), late steps
+    pinned = [tuple(torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).pin_memory() for x in host_steps[t])
+              for t in range(wl.n_discovery, min(wl.steps, wl.n_discovery + 4))]
+    O_host = torch.empty(O.shape, dtype=torch.bfloat16).pin_memory()
+    Qd, Kd, Vd = (torch.empty_like(x) for x in dev_steps[0])
+    h2d = sum(x.numel() * x.element_size() for x in pinned[0])
+    d2h = O_host.numel() * O_host.element_size()
+    e2e_iters = max(8, args.steps)
+    e_start, e_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    torch.cuda.synchronize()
+    e_start.record(stream)
+    for i in range(e2e_iters):
+        hq, hk, hv = pinned[i % len(pinned)]
+        Qd.copy_(hq, non_blocking=True)
+        Kd.copy_(hk, non_blocking=True)
+        Vd.copy_(hv, non_blocking=True)
+        wise.wise_sparse_attn(shape, Qd, Kd, Vd, layer.idx, layer.counts, O)
+        O_host.copy_(O, non_blocking=True)
+    e_end.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e_start.elapsed_time(e_end) / e2e_iters
+    clk = clocks.stop()
+    status = wise.wise_get_status()
+    if status != wise.WISE_OK:
+        raise RuntimeError(f"kernel status: {wise.status_string(status)}")
+
+    value = statistics.mean(late_only)
+    dense = statistics.mean(dense_ms)
+    per_rank = torch.tensor([value, total_ms / args.steps, e2e_ms], dtype=torch.float64, device="cuda")
+    if world > 1:
+        dist.all_reduce(per_rank, op=dist.ReduceOp.MAX)
+    value, step_ms, e2e_ms = (float(x) for x in per_rank.tolist())
+
+    peaks, peak_kind = load_peaks()
+    peak = float(peaks["bf16_tflops"])
+    achieved = flops_sparse / (value * 1e-3) / 1e12
+    launches = args.steps * (wl.steps + 1)  # n_discovery dense + 1 select + n_late sparse per trajectory
+
+    line = {
+        "metric": "late-step attention ms/step (sparse, 4K)",
+        "value": round(value, 5),
+        "unit": "ms",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(step_ms, 4),
+        "higher_is_better": False,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": "4k: batch 1, L=4096, 32 heads, head_dim 128, block 128, T=32, discovery 0-3, "
+                               "sink+diagonal+95% coverage cap 8",
+                   "step": "one T=32 trajectory: 4 dense+mass, 1 selection, 28 sparse",
+                   "l2": "every recurrent step has its own Q/K/V (2.9 GB rotating, > L2)",
+                   "parallelism": f"replicas x{world}"},
+        "dense_ms": round(dense, 5),
+        "speedup_vs_dense": round(dense / value, 4),
+        "setup_inclusive_speedup": round(n_late * dense / (statistics.mean(sel_ms) + n_late * value), 4),
+        "trajectory_speedup": round(wl.steps * dense / step_ms, 4),
+        "discovery_ms": round(statistics.mean(disc_ms), 5),
+        "select_ms": round(statistics.mean(sel_ms), 5),
+        "tflops_effective": round(achieved, 2),
+        "dense_tflops": round(flops_dense / (dense * 1e-3) / 1e12, 2),
+        "density": round(density, 4),
+        "roofline": {"bound": "tensor", "achieved": round(achieved, 2), "peak": peak, "unit": "TFLOP/s",
+                     "frac": round(achieved / peak, 4), "traffic": None,
+                     "peak_kind": f"{peak_kind} bf16 burst", "kernel": "wise_sparse_attn"},
+        "e2e": {"value": round(e2e_ms, 5), "unit": "ms", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": launches,
+        "clocks": clk,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        ms, cores, sec = oracle_late_step_ms(wl, host_steps[wl.n_discovery], idx_h, counts_h, 4)
+        line["cpu_baseline"] = {"value": round(ms, 1), "unit": "ms", "cores": cores, "kind": "oracle",
+                                "sample": f"4 of 32 heads of one late step ({sec:.1f} s), scaled x8"}
+    if rank == 0:
+        print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,138 @@
+/*
+ * wise.h -- C ABI of the WISE attention hot path on GB300 (sm_103a).
+ *
+ * WISE (working-set inference with support exploitation) runs a
+ * recurrent-depth transformer's attention in two phases (Sec. 5):
+ *   discovery  dense causal attention (Eq. 2) whose block attention mass
+ *              (Eq. 5) is accumulated over the early recurrent steps;
+ *   selection  the accumulated mass is turned, once, into a per-(batch,
+ *              kv-head, query-block) list of key blocks (Eq. 6);
+ *   reuse      late steps recompute Q, K, V and the softmax, restricted to
+ *              that fixed block support (Eqs. 7-8).
+ * Each entry point below is one hand-written CUDA kernel.
+ *
+ * Conventions shared by all entry points
+ *  - Tensors are dense, contiguous, row-major device buffers owned by the
+ *    caller.  Q and O are [batch, n_heads, seqlen, head_dim] bf16; K and V are
+ *    [batch, n_kv_heads, seqlen, head_dim] bf16.  Query head h reads kv-head
+ *    h / (n_heads / n_kv_heads) (grouped-query attention).
+ *  - Q/K/V/O must be 16-byte aligned, blockmass/idx/counts 4-byte aligned.
+ *  - head_dim is 64, 96 or 128; block (B) is 64 or 128; seqlen % block == 0.
+ *    nQB = nKB = seqlen / block.
+ *  - Every call is asynchronous on `stream` and returns a status code
+ *    (WISE_OK or a negative WISE_ERR_*) describing argument checks and the
+ *    launch; nothing is done when a check fails.  Faults found by a kernel
+ *    while it runs (an inconsistent support list, an internal wait that ran
+ *    out) are recorded in a per-device status word read by wise_get_status().
+ *  - Empty problems (batch == 0 or seqlen == 0) return WISE_OK and launch
+ *    nothing.
+ *  - Inputs are never written.  The library keeps one lazily allocated
+ *    scratch buffer per device for the block-mass epilogue (see
+ *    wise_full_attn_accumulate); no other call allocates device memory.
+ */
+#ifndef WISE_H_
+#define WISE_H_
+
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define WISE_OK 0
+#define WISE_ERR_INVALID_ARG -1 /* NULL or misaligned pointer, negative size, bad selection parameters */
+#define WISE_ERR_UNSUPPORTED -2 /* head_dim / block / head grouping / device not supported */
+#define WISE_ERR_SHAPE -3       /* seqlen not a multiple of block */
+#define WISE_ERR_CUDA -4        /* a CUDA runtime call or kernel launch failed */
+#define WISE_ERR_TIMEOUT -5     /* a kernel's internal wait ran out (reported by wise_get_status) */
+#define WISE_ERR_BAD_SUPPORT -6 /* idx/counts held entries outside the rules (reported by wise_get_status) */
+
+#define WISE_SEL_TOPK 0
+#define WISE_SEL_COVERAGE 1
+
+/* Problem geometry (Sec. 3: n = seqlen, d_h = head_dim; Sec. 5.1: block B). */
+typedef struct {
+  int batch;
+  int seqlen;
+  int n_heads;    /* query heads */
+  int n_kv_heads; /* key/value heads; n_heads % n_kv_heads == 0 */
+  int head_dim;
+  int block;
+  float scale;    /* softmax scale; 0 selects 1/sqrt(head_dim) as in Eq. 2 */
+} wise_shape_t;
+
+/* Support-selection rule (Eq. 6, single-pass form).
+ * For query block q the admissible key blocks are 0..q.  Forced blocks:
+ * 0..n_sink-1 and q-n_local+1..q (clipped to 0..q).  The remaining blocks are
+ * ranked by pooled fixed-point mass (descending; ties to the lower index) and
+ * added in rank order:
+ *   WISE_SEL_TOPK      the first `topk` of them;
+ *   WISE_SEL_COVERAGE  until the kept mass reaches eta of the admissible
+ *                      mass (the cumulative-mass support of Eq. 6);
+ * never exceeding `cap` blocks in total, forced ones included. */
+typedef struct {
+  int n_sink;  /* >= 0 */
+  int n_local; /* >= 1 (1 = diagonal block only) */
+  int mode;    /* WISE_SEL_TOPK or WISE_SEL_COVERAGE */
+  int topk;    /* >= 0, used by WISE_SEL_TOPK */
+  float eta;   /* in [0, 1], used by WISE_SEL_COVERAGE */
+  int cap;     /* >= n_sink + n_local; width of each idx row */
+} wise_select_t;
+
+/* Dense causal attention of one recurrent step, with the block attention
+ * mass of that step accumulated on the fly.
+ *   O = softmax(Q K^T * scale + M) V, M causal                      (Eq. 2)
+ *   r_qb = (1/B) sum_{i in I_q} sum_{j in I_b} A_ij                  (Eq. 5)
+ *   blockmass[b,h,q,kb] = (step == 0 ? 0 : blockmass[b,h,q,kb]) + r_qkb
+ * blockmass is fp32 [batch, n_heads, nQB, nKB] (per query head; entries with
+ * kb > q are written as 0 when step == 0 and left as they are otherwise).
+ * blockmass == NULL runs plain dense attention (the dense baseline) and
+ * ignores `step`.  Accumulation with step > 0 is a read-modify-write: calls on
+ * the same blockmass must be ordered on the stream.
+ * The first call with blockmass != NULL on a device allocates the library's
+ * scratch buffer (and grows it when a later shape needs more); make that
+ * first call outside any CUDA-graph capture. */
+int wise_full_attn_accumulate(const wise_shape_t* shape, const void* Q, const void* K, const void* V, void* O,
+                              float* blockmass, int step, cudaStream_t stream);
+
+/* Support selection from accumulated block mass (Eq. 6, rule of
+ * wise_select_t).  Masses of the query heads of each kv-head group are pooled
+ * in exact fixed point, u(x) = floor(min(x, 4096) * 2^32) for x > 0 (else 0),
+ * so the result is a deterministic function of the fp32 input; coverage
+ * compares cum * 65536 >= floor(eta * 65536 + 0.5) * total exactly.
+ * blockmass: fp32 [batch, n_heads, nQB, nKB], entries kb <= q are read.
+ * idx:    int32 [batch, n_kv_heads, nQB, cap], ascending block ids, -1 padded.
+ * counts: int32 [batch, n_kv_heads, nQB]. */
+int wise_select_support(const wise_shape_t* shape, const wise_select_t* sel, const float* blockmass,
+                        int32_t* idx, int32_t* counts, cudaStream_t stream);
+
+/* Attention of one late recurrent step restricted to the block support
+ *   R_ij = 0 if b(j) in B_q(i) else -inf                              (Eq. 7)
+ *   O = softmax(Q K^T * scale + M + R) V, M causal                    (Eq. 8)
+ * Q, K, V are the current step's (recomputed every step, Sec. 5.2); idx and
+ * counts are wise_select_support's output (row width `cap`).  Query head h
+ * uses the support of kv-head h / (n_heads / n_kv_heads).  Within each row the
+ * first counts entries are used; they must be ascending block ids in
+ * [0, q].  Entries that break this are skipped and flagged as
+ * WISE_ERR_BAD_SUPPORT in the status word.  A query row with no admissible key
+ * gets O = 0. */
+int wise_sparse_attn(const wise_shape_t* shape, const void* Q, const void* K, const void* V, const int32_t* idx,
+                     const int32_t* counts, int cap, void* O, cudaStream_t stream);
+
+/* Synchronizes `stream`, then reads and clears the current device's status
+ * word: WISE_OK, WISE_ERR_BAD_SUPPORT or WISE_ERR_TIMEOUT (the latter wins
+ * when both were recorded), or WISE_ERR_CUDA if the synchronization failed. */
+int wise_get_status(cudaStream_t stream);
+
+/* Static description of a status code. */
+const char* wise_status_string(int status);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int wise_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* WISE_H_ */

@@ -1,0 +1,57 @@
+// Declarations shared by the translation units of libwise.so.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace wise {
+
+enum AttnMode : int { kDense = 0, kDenseMass = 1, kSparse = 2 };
+
+// Bits of the per-device status word.
+constexpr int kStatusTimeout = 1;
+constexpr int kStatusBadSupport = 2;
+
+struct AttnParams {
+  int batch, seqlen, n_heads, n_kv_heads, group;
+  int n_qtiles;   // ceil(seqlen / 128): 128-row query tiles
+  int n_blocks;   // nQB = nKB = seqlen / block
+  int n_units;    // batch * n_heads * n_qtiles
+  float scale_log2;
+  __nv_bfloat16* O;
+  float* blockmass;       // kDenseMass
+  int step;               // kDenseMass: 0 overwrites, > 0 accumulates
+  const int32_t* idx;     // kSparse
+  const int32_t* counts;  // kSparse
+  int cap;                // kSparse
+  float* scratch;         // kDenseMass: [gridDim.x][n_blocks][128] log2 partial masses
+  int* status;
+};
+
+struct AttnLaunch {
+  CUtensorMap mapQ, mapK, mapV;
+  AttnParams p;
+  int grid;
+  cudaStream_t stream;
+};
+
+// Defined in attn_d64.cu / attn_d96.cu / attn_d128.cu.
+cudaError_t launch_attn_d64(int block, int mode, const AttnLaunch& L);
+cudaError_t launch_attn_d96(int block, int mode, const AttnLaunch& L);
+cudaError_t launch_attn_d128(int block, int mode, const AttnLaunch& L);
+
+struct SelectParams {
+  int batch, n_heads, n_kv_heads, group, n_blocks;
+  int n_sink, n_local, mode, topk, cap;
+  uint64_t eta16;  // floor(eta * 65536 + 0.5)
+  const float* blockmass;
+  int32_t* idx;
+  int32_t* counts;
+};
+
+// Defined in select.cu.
+cudaError_t launch_select(const SelectParams& p, cudaStream_t stream);
+
+}  // namespace wise

@@ -174,12 +174,14 @@ class Trajectory:
         return tuple(f32_to_bf16_bits(X) for X in self.state)
 
 
-def random_qkv(batch, n_heads, n_kv_heads, seqlen, head_dim, seed, std=1.0):
-    """Plain N(0, std^2) bf16 Q/K/V (no planted routing)."""
+def random_qkv(batch, n_heads, n_kv_heads, seqlen, head_dim, seed, std=1.0, v_std=None):
+    """Plain bf16 Q/K ~ N(0, std^2), V ~ N(0, v_std^2) (v_std defaults to std);
+    no planted routing."""
     rng = np.random.default_rng(seed)
+    v_std = std if v_std is None else v_std
     Q = rng.standard_normal((batch, n_heads, seqlen, head_dim), dtype=np.float32) * np.float32(std)
     K = rng.standard_normal((batch, n_kv_heads, seqlen, head_dim), dtype=np.float32) * np.float32(std)
-    V = rng.standard_normal((batch, n_kv_heads, seqlen, head_dim), dtype=np.float32) * np.float32(std)
+    V = rng.standard_normal((batch, n_kv_heads, seqlen, head_dim), dtype=np.float32) * np.float32(v_std)
     return f32_to_bf16_bits(Q), f32_to_bf16_bits(K), f32_to_bf16_bits(V)
 
 
