@@ -96,6 +96,39 @@ typedef struct {
 int wise_full_attn_accumulate(const wise_shape_t* shape, const void* Q, const void* K, const void* V, void* O,
                               float* blockmass, int step, cudaStream_t stream);
 
+/* Capacity of the fixed scratch array used by
+ * wise_full_attn_accumulate_noalloc (8 MiB per device). */
+#define WISE_NOALLOC_SCRATCH_BYTES (8u << 20)
+
+/* wise_full_attn_accumulate with a non-NULL blockmass, for callers that
+ * cannot have this library allocate device memory.  The paper has no
+ * counterpart: this is a deployment variant of the same kernel.
+ *
+ * Who needs it: a process whose device memory is handed out by another
+ * allocator (a framework's caching allocator that has reserved the pool, a
+ * fixed memory budget), or a serving loop that cannot afford the device-wide
+ * synchronisation cudaMalloc/cudaFree may cause while other streams run.
+ * wise_full_attn_accumulate obtains its scratch with cudaMalloc on first use
+ * (and frees and reallocates it when a larger problem comes); this entry
+ * point calls neither cudaMalloc nor cudaFree nor any allocating routine.
+ * Its scratch is a fixed array of WISE_NOALLOC_SCRATCH_BYTES compiled into
+ * the library, held by every device that loads the library until the
+ * process exits.
+ *
+ * Arguments, layouts and results are those of wise_full_attn_accumulate;
+ * blockmass must not be NULL (plain dense attention uses no scratch).
+ * Limit: one call needs min(batch*n_heads*ceil(seqlen/128), SM count) *
+ * nKB * 512 bytes of scratch; larger problems return WISE_ERR_UNSUPPORTED and
+ * launch nothing.  On a 152-SM GB300 with at least 152 query tiles that is
+ * nKB <= 107 (seqlen <= 13696 with block 128).
+ * The first call on each device looks up the array's device address (with
+ * that device current) and caches it; make that first call before any CUDA
+ * stream capture.  All calls on a device share the one array: calls whose
+ * kernels can run at the same time on that device (unordered streams) race
+ * on it and corrupt each other's block mass. */
+int wise_full_attn_accumulate_noalloc(const wise_shape_t* shape, const void* Q, const void* K, const void* V,
+                                      void* O, float* blockmass, int step, cudaStream_t stream);
+
 /* Support selection from accumulated block mass (Eq. 6, rule of
  * wise_select_t).  Masses of the query heads of each kv-head group are pooled
  * in exact fixed point, u(x) = floor(min(x, 4096) * 2^32) for x > 0 (else 0),

@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "wise.h"
+
 namespace wise {
 
 enum AttnMode : int { kDense = 0, kDenseMass = 1, kSparse = 2 };
@@ -50,6 +52,15 @@ struct SelectParams {
   int32_t* idx;
   int32_t* counts;
 };
+
+// Argument checks, tensor maps and launch of the attention kernels (defined
+// in wise_api.cu).  For kDenseMass the per-CTA scratch comes from the
+// library's lazily allocated per-device buffer, unless caller_scratch is
+// given: then that device buffer of caller_scratch_bytes is used and a
+// problem needing more returns WISE_ERR_UNSUPPORTED.
+int launch_attention(const wise_shape_t* sh, const void* Q, const void* K, const void* V, void* O, int mode,
+                     float* blockmass, int step, const int32_t* idx, const int32_t* counts, int cap,
+                     cudaStream_t stream, float* caller_scratch = nullptr, size_t caller_scratch_bytes = 0);
 
 // Defined in select.cu.
 cudaError_t launch_select(const SelectParams& p, cudaStream_t stream);

@@ -123,9 +123,11 @@ bool make_map(CUtensorMap* map, const void* base, int head_dim, int seqlen, long
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+}  // namespace
+
 int launch_attention(const wise_shape_t* sh, const void* Q, const void* K, const void* V, void* O, int mode,
                      float* blockmass, int step, const int32_t* idx, const int32_t* counts, int cap,
-                     cudaStream_t stream) {
+                     cudaStream_t stream, float* caller_scratch, size_t caller_scratch_bytes) {
   int rc = check_shape(sh, true);
   if (rc != WISE_OK) return rc;
   if (sh->batch == 0 || sh->seqlen == 0) return WISE_OK;
@@ -176,8 +178,14 @@ int launch_attention(const wise_shape_t* sh, const void* Q, const void* K, const
   L.stream = stream;
   p.scratch = nullptr;
   if (mode == kDenseMass) {
-    p.scratch = scratch_at_least(ds, (size_t)L.grid * n_blocks * 128 * sizeof(float));
-    if (!p.scratch) return WISE_ERR_CUDA;
+    const size_t need = (size_t)L.grid * n_blocks * 128 * sizeof(float);
+    if (caller_scratch) {
+      if (need > caller_scratch_bytes) return WISE_ERR_UNSUPPORTED;
+      p.scratch = caller_scratch;
+    } else {
+      p.scratch = scratch_at_least(ds, need);
+      if (!p.scratch) return WISE_ERR_CUDA;
+    }
   }
   cudaError_t e;
   switch (sh->head_dim) {
@@ -188,7 +196,6 @@ int launch_attention(const wise_shape_t* sh, const void* Q, const void* K, const
   return e == cudaSuccess ? WISE_OK : WISE_ERR_CUDA;
 }
 
-}  // namespace
 }  // namespace wise
 
 using namespace wise;

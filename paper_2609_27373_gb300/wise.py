@@ -26,8 +26,9 @@ WISE_ERR_BAD_SUPPORT = -6
 WISE_SEL_TOPK = 0
 WISE_SEL_COVERAGE = 1
 
-EXPORTS = ("wise_full_attn_accumulate", "wise_select_support", "wise_sparse_attn", "wise_get_status",
-           "wise_status_string", "wise_version")
+EXPORTS = ("wise_full_attn_accumulate", "wise_full_attn_accumulate_noalloc", "wise_select_support",
+           "wise_sparse_attn", "wise_get_status", "wise_status_string", "wise_version")
+NOALLOC_SCRATCH_BYTES = 8 << 20
 
 
 class WiseError(RuntimeError):
@@ -96,6 +97,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib = ctypes.CDLL(path)
         P = ctypes.c_void_p
         lib.wise_full_attn_accumulate.argtypes = [ctypes.POINTER(wise_shape_t), P, P, P, P, P, ctypes.c_int, P]
+        lib.wise_full_attn_accumulate_noalloc.argtypes = [ctypes.POINTER(wise_shape_t), P, P, P, P, P, ctypes.c_int,
+                                                          P]
         lib.wise_select_support.argtypes = [ctypes.POINTER(wise_shape_t), ctypes.POINTER(wise_select_t), P, P, P, P]
         lib.wise_sparse_attn.argtypes = [ctypes.POINTER(wise_shape_t), P, P, P, P, P, ctypes.c_int, P, P]
         lib.wise_get_status.argtypes = [P]
@@ -155,6 +158,22 @@ def wise_full_attn_accumulate(shape: Shape, Q, K, V, O, blockmass=None, step: in
                                           int(step), _stream(stream))
     if rc != WISE_OK:
         raise WiseError(rc, "wise_full_attn_accumulate")
+
+
+def wise_full_attn_accumulate_noalloc(shape: Shape, Q, K, V, O, blockmass, step: int = 0, stream=None) -> None:
+    """wise_full_attn_accumulate with block mass, without any device
+    allocation by the library: its scratch is a fixed 8 MiB array compiled
+    into libwise.so.  For callers whose device memory is managed elsewhere or
+    who cannot afford cudaMalloc's synchronisation; problems whose scratch
+    would exceed the array are rejected (WiseError, WISE_ERR_UNSUPPORTED)."""
+    _qkvo(shape, Q, K, V, O)
+    nb = shape.n_blocks
+    _check(blockmass, "blockmass", (shape.batch, shape.n_heads, nb, nb), torch.float32)
+    sh = shape.c()
+    rc = load().wise_full_attn_accumulate_noalloc(ctypes.byref(sh), _ptr(Q), _ptr(K), _ptr(V), _ptr(O),
+                                                  _ptr(blockmass), int(step), _stream(stream))
+    if rc != WISE_OK:
+        raise WiseError(rc, "wise_full_attn_accumulate_noalloc")
 
 
 def wise_select_support(shape: Shape, sel: Select, blockmass, idx, counts, stream=None) -> None:
