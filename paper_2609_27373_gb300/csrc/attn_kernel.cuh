@@ -4,38 +4,57 @@
 //               accumulated into blockmass
 //   kSparse     key blocks restricted to the selected support      (Eqs. 7-8)
 //
-// Work decomposition.  A unit is one 128-row query tile of one (batch, head).
-// The grid is persistent (one CTA per SM); CTA c takes units c, c + grid, ...
-// in order of decreasing causal length.  Each unit walks its list of key
-// tiles (BN = block keys each): every tile of the causal prefix (dense), or
-// the blocks of the support (sparse; with block 64 a query tile covers two
-// query blocks and walks the union of their lists, masking per half).
+// Work decomposition.  A unit is one 128-row query tile of one (batch, head);
+// units are numbered in order of decreasing causal length, and the
+// persistent grid (one CTA per SM) hands CTA c the units c, c + grid, ...
+// Each unit walks its list of key tiles (BN = block keys each): every tile of
+// the causal prefix (dense), or the blocks of the support (sparse; with block
+// 64 a query tile covers two query blocks and walks the union of their lists,
+// masking per half).
 //
-// Warp roles (192 threads):
-//   warps 0-3  softmax: thread t owns query row t of the tile (= TMEM lane t).
-//              It reads its row of S from TMEM, keeps the running max and sum
-//              (online softmax in the log2 domain, with the rescale of O
-//              skipped unless the max grows by more than 2^8), writes P as
-//              bf16 into shared memory, and runs the epilogue: O / l to
-//              global memory, and for kDenseMass the block masses.
-//   warp 4     TMA producer: Q tile (double-buffered across units) and K/V
-//              tiles (kStages-deep ring).
-//   warp 5     MMA issuer: S = Q K^T into one of two TMEM S buffers, then
-//              O += P V into the TMEM O accumulator, one tile behind, so the
-//              tensor core computes S(j+1) while the softmax works on S(j).
+// Both products run with the A operand in tensor memory, because a tcgen05
+// MMA that reads both operands from shared memory is limited by the shared
+// memory read rate to about half the tensor peak (measured: 118 clk per
+// M128/N128/K16 step with both operands in shared memory, 66 clk with A in
+// TMEM):
+//   S = Q K^T    Q copied once per unit from shared memory into TMEM, K
+//                from shared memory (K-major);
+//   O += P V     P written by the softmax into TMEM, V from shared memory
+//                (MN-major).
+// TMEM (512 columns): Q double-buffered across units (2 x 64 columns), S
+// double-buffered across tiles (2 x 128 columns, P overwrites the first BN/2
+// columns of its S), O (128 columns).
 //
-// Block mass (Eq. 5) needs each row's final normaliser, which is known only
-// after the last tile.  For every tile the softmax thread stores
-// lc = m + log2(sum_{j in tile} 2^(s_j - m)) (its row's partial mass in log2
-// units, m the running max at the time) in a per-CTA scratch row; the
-// epilogue turns it into A-mass 2^(lc - lse), sums the 128 (or 2 x 64) rows
-// of each query block with warp shuffles and a fixed-order cross-warp sum
-// (deterministic), divides by B and writes or accumulates blockmass.
+// Warp roles (352 threads):
+//   warps 0-3 and 4-7  two softmax warpgroups.  Thread t of warpgroup h owns
+//              query row t (= TMEM lane t), key columns [h BN/2, (h+1) BN/2)
+//              of every S tile and output columns [h D/2, (h+1) D/2) of O.
+//              Per tile it loads its half row of S, exchanges the half-row
+//              maximum with its partner thread (bounded mbarrier), keeps the
+//              running max and its half of the row sum (online softmax in the
+//              log2 domain; O is rescaled only when the max grows by more than
+//              2^8), and writes its half of P into TMEM.  Per unit it copies
+//              the next unit's Q into TMEM and runs the epilogue: O / l to
+//              global memory and, for kDenseMass, the block masses.
+//   warp 8     TMA producer: K tiles into a ring of kRingK entries and V tiles
+//              into a ring of kRingV entries, in the order K(0), K(1), V(0),
+//              K(2), V(1), ...
+//   warp 9     S issuer: S(j) = Q K(j)^T into S buffer j & 1, one tile ahead
+//              of the softmax.
+//   warp 10    P V issuer: O += P(j) V(j) once the softmax has written P(j).
+//   A tcgen05.mma issue blocks its thread while the tensor core drains the
+//   previous instructions, so the two products are issued from two threads:
+//   each thread's barrier checks overlap the other's issue and the tensor
+//   core stays fed.  S(j) reuses the buffer of P(j-2); the P V thread commits
+//   buf_free[b] after each P V so that the S thread can wait for it.
+//
 #pragma once
 
 #include <cuda_bf16.h>
 #include <limits.h>
 #include <stdint.h>
+
+#include <type_traits>
 
 #include "internal.cuh"
 #include "ptx.cuh"
@@ -45,19 +64,31 @@ namespace wise {
 template <int D, int BN>
 struct AttnCfg {
   static constexpr int kBoxes = (D + 63) / 64;          // 64-column TMA boxes per row tile
-  static constexpr int kQBytes = kBoxes * 128 * 128;    // one 128-row Q tile
-  static constexpr int kKVBytes = kBoxes * BN * 128;    // one BN-row K or V tile
-  static constexpr int kPBytes = (BN / 64) * 128 * 128; // P tile, 128 x BN bf16
-  static constexpr int kStages = (D <= 64) ? 4 : 2;
-  static constexpr int kSmemBytes = 2 * kQBytes + 2 * kStages * kKVBytes + kPBytes + 1024;
+  static constexpr int kQBytes = kBoxes * 128 * 128;    // one 128-row Q tile (staging)
+  static constexpr int kKVBytes = kBoxes * BN * 128;    // one BN-row K or V tile (one ring entry)
+  // Dynamic shared memory available after the 1024-byte alignment slack and
+  // the static barriers and exchange buffers.
+  static constexpr int kBudget = 227 * 1024 - 1024 - 2560;
+  static constexpr int kRingFit = (kBudget - kQBytes) / kKVBytes;
+  static constexpr int kRing = kRingFit > 12 ? 12 : kRingFit;
+  static constexpr int kRingK = (kRing + 1) / 2;  // K tiles (consumed by S)
+  static constexpr int kRingV = kRing / 2;        // V tiles (consumed by P V)
+  static constexpr int kSmemBytes = kQBytes + kRing * kKVBytes + 1024;
   // At least 116 KB so that a single CTA resides per SM (it owns all 512
   // TMEM columns).
   static constexpr int kSmemLaunch = kSmemBytes > 116 * 1024 ? kSmemBytes : 116 * 1024;
-  static constexpr uint32_t kTmemO = 2 * BN;            // S buffers at columns 0 and BN
+  static constexpr uint32_t kTmemQ = 0;       // two Q buffers
+  static constexpr uint32_t kTmemQCols = 64;  // 128 bf16 of Q per row
+  static constexpr uint32_t kTmemS = 128;     // two S/P buffers
+  static constexpr uint32_t kTmemSCols = 128;
+  static constexpr uint32_t kTmemO = 384;     // O accumulator
   static constexpr uint32_t kTmemCols = 512;
-  static constexpr int kThreads = 192;
-  static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
-  static_assert(2 * BN + D <= 512, "TMEM budget");
+  static constexpr int kThreads = 352;
+  static constexpr int kProducerWarp = 8;
+  static constexpr int kMmaSWarp = 9;   // issues S = Q K^T, owns the TMEM allocation
+  static constexpr int kMmaPVWarp = 10; // issues O += P V
+  static_assert(kRingV >= 1 && kRingK >= 2, "shared memory budget");
+  static_assert(BN <= 128 && D <= 128, "TMEM budget");
 };
 
 __device__ __forceinline__ float ex2_approx(float x) {
@@ -77,11 +108,13 @@ __device__ __forceinline__ float lg2_approx(float x) {
 // lists of its two query blocks (block 64); `bits` says which half of the
 // 128 query rows may attend the tile.  Entries that are negative, beyond the
 // query block, or not strictly ascending are skipped and flagged in `bad`.
+// Fields a variant does not use are never touched, so they cost no registers.
+template <int BN, int MODE>
 struct TileIter {
-  int dense, cur, last;
-  const int32_t* la;
-  const int32_t* lb;
+  int cur, last;                                   // dense
+  const int32_t* la;                               // sparse, first query block
   int na, ia, lima, preva, pend_a;
+  const int32_t* lb;                               // sparse, second query block (block 64)
   int nb, ib, limb, prevb, pend_b;
   int bad;
 
@@ -99,28 +132,35 @@ struct TileIter {
   }
 
   __device__ __forceinline__ bool next(int& kb, int& bits) {
-    if (dense) {
+    if constexpr (MODE != kSparse) {
       if (cur > last) return false;
       kb = cur++;
       bits = 3;
       return true;
-    }
-    if (pend_a == INT_MAX && pend_b == INT_MAX) return false;
-    if (pend_a < pend_b) {
+    } else if constexpr (BN == 128) {
+      if (pend_a == INT_MAX) return false;
       kb = pend_a;
       bits = 1;
       pend_a = pull(la, na, ia, lima, preva);
-    } else if (pend_b < pend_a) {
-      kb = pend_b;
-      bits = 2;
-      pend_b = pull(lb, nb, ib, limb, prevb);
+      return true;
     } else {
-      kb = pend_a;
-      bits = 3;
-      pend_a = pull(la, na, ia, lima, preva);
-      pend_b = pull(lb, nb, ib, limb, prevb);
+      if (pend_a == INT_MAX && pend_b == INT_MAX) return false;
+      if (pend_a < pend_b) {
+        kb = pend_a;
+        bits = 1;
+        pend_a = pull(la, na, ia, lima, preva);
+      } else if (pend_b < pend_a) {
+        kb = pend_b;
+        bits = 2;
+        pend_b = pull(lb, nb, ib, limb, prevb);
+      } else {
+        kb = pend_a;
+        bits = 3;
+        pend_a = pull(la, na, ia, lima, preva);
+        pend_b = pull(lb, nb, ib, limb, prevb);
+      }
+      return true;
     }
-    return true;
   }
 };
 
@@ -133,38 +173,32 @@ __device__ __forceinline__ int clamp_count(int n, int cap, int& bad) {
 }
 
 template <int BN, int MODE>
-__device__ __forceinline__ TileIter make_iter(const AttnParams& p, int b, int kvh, int qt) {
-  TileIter it;
+__device__ __forceinline__ TileIter<BN, MODE> make_iter(const AttnParams& p, int b, int kvh, int qt) {
+  TileIter<BN, MODE> it;
   it.bad = 0;
-  if (MODE != kSparse) {
-    it.dense = 1;
+  if constexpr (MODE != kSparse) {
     it.cur = 0;
     const int last_row = min(qt * 128 + 127, p.seqlen - 1);
     it.last = last_row / BN;
-    it.pend_a = it.pend_b = INT_MAX;
-    return it;
-  }
-  it.dense = 0;
-  constexpr int kQbPerTile = 128 / BN;
-  const int q0 = qt * kQbPerTile;
-  const size_t row0 = ((size_t)b * p.n_kv_heads + kvh) * p.n_blocks + q0;
-  it.la = p.idx + row0 * p.cap;
-  it.na = clamp_count(__ldg(p.counts + row0), p.cap, it.bad);
-  it.ia = 0;
-  it.lima = q0;
-  it.preva = -1;
-  if (kQbPerTile == 2 && q0 + 1 < p.n_blocks) {
-    it.lb = p.idx + (row0 + 1) * p.cap;
-    it.nb = clamp_count(__ldg(p.counts + row0 + 1), p.cap, it.bad);
   } else {
-    it.lb = it.la;
-    it.nb = 0;
+    constexpr int kQbPerTile = 128 / BN;
+    const int q0 = qt * kQbPerTile;
+    const size_t row0 = ((size_t)b * p.n_kv_heads + kvh) * p.n_blocks + q0;
+    it.la = p.idx + row0 * p.cap;
+    it.na = clamp_count(__ldg(p.counts + row0), p.cap, it.bad);
+    it.ia = 0;
+    it.lima = q0;
+    it.preva = -1;
+    it.pend_a = it.pull(it.la, it.na, it.ia, it.lima, it.preva);
+    if constexpr (kQbPerTile == 2) {
+      it.lb = p.idx + (row0 + 1) * p.cap;
+      it.nb = (q0 + 1 < p.n_blocks) ? clamp_count(__ldg(p.counts + row0 + 1), p.cap, it.bad) : 0;
+      it.ib = 0;
+      it.limb = q0 + 1;
+      it.prevb = -1;
+      it.pend_b = it.pull(it.lb, it.nb, it.ib, it.limb, it.prevb);
+    }
   }
-  it.ib = 0;
-  it.limb = q0 + 1;
-  it.prevb = -1;
-  it.pend_a = it.pull(it.la, it.na, it.ia, it.lima, it.preva);
-  it.pend_b = it.pull(it.lb, it.nb, it.ib, it.limb, it.prevb);
   return it;
 }
 
@@ -176,12 +210,78 @@ __device__ __forceinline__ void decode_unit(const AttnParams& p, int u, int& b, 
   h = bh % p.n_heads;
 }
 
+// One key tile of the CTA's stream, as the producer and the MMA warp need it.
+struct Tile {
+  int kb;     // key block
+  int z;      // batch * n_kv_heads + kv head (TMA outer coordinate of K and V)
+  int first;  // first tile of its unit
+};
+
+// The tiles of one CTA, unit after unit (units without any tile skipped).
+template <int BN, int MODE>
+struct TileStream {
+  int u, stride, z;
+  TileIter<BN, MODE> it;
+  int nkb, nfirst, have;
+  int bad;
+
+  __device__ __forceinline__ void open_next_unit(const AttnParams& p) {
+    for (;;) {
+      u += stride;
+      if (u >= p.n_units) {
+        have = 0;
+        return;
+      }
+      int b, h, qt;
+      decode_unit(p, u, b, h, qt);
+      const int kvh = h / p.group;
+      z = b * p.n_kv_heads + kvh;
+      it = make_iter<BN, MODE>(p, b, kvh, qt);
+      int bits;
+      if (it.next(nkb, bits)) {
+        nfirst = 1;
+        have = 1;
+        return;
+      }
+      bad |= it.bad;
+    }
+  }
+
+  __device__ __forceinline__ void start(const AttnParams& p) {
+    stride = gridDim.x;
+    u = blockIdx.x - stride;
+    bad = 0;
+    open_next_unit(p);
+  }
+
+  __device__ __forceinline__ bool next(const AttnParams& p, Tile& t) {
+    if (!have) return false;
+    t.kb = nkb;
+    t.z = z;
+    t.first = nfirst;
+    int bits;
+    if (it.next(nkb, bits)) {
+      nfirst = 0;
+    } else {
+      bad |= it.bad;
+      open_next_unit(p);
+    }
+    return true;
+  }
+};
+
+template <int RK, int RV>
 struct SharedBarriers {
-  uint64_t q_full[2], q_empty[2];
-  uint64_t k_full[4], v_full[4], kv_empty[4];
-  uint64_t s_full[2];
-  uint64_t p_full, o_full, mma_done;
-  uint64_t epi;  // the four softmax warps meet here in the block-mass epilogue
+  uint64_t k_full[RK], k_empty[RK], v_full[RV], v_empty[RV];
+  uint64_t q_full;       // Q tile landed in the staging buffer (TMA)
+  uint64_t q_tmem;       // Q tile copied into TMEM (8 softmax warps)
+  uint64_t s_full[2];    // S buffer b written (S thread commit)
+  uint64_t buf_free[2];  // P of buffer b consumed by its P V (P V thread commit)
+  uint64_t p_full;       // P written into TMEM (8 softmax warps)
+  uint64_t o_full;       // a P V completed (P V thread commit)
+  uint64_t xch;          // the two softmax halves exchanged row values (8 warps)
+  uint64_t s_done, pv_done;
+  float xbuf[2][2][128];  // [phase & 1][half][row]
   uint32_t tmem_base;
   int abort;
 };
@@ -192,204 +292,297 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
   return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort));
 }
 
-__device__ __forceinline__ void raise_status(const AttnParams& p, SharedBarriers& sb, int bits) {
-  sb.abort = 1;
+__device__ __forceinline__ void raise_status(const AttnParams& p, int* abort, int bits) {
+  *reinterpret_cast<volatile int*>(abort) = 1;
   atomicOr(p.status, bits);
 }
 
 // ------------------------------------------------------------------ producer
 template <int D, int BN, int MODE>
-__device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, const CUtensorMap* mapV,
-                              const AttnParams& p, uint8_t* sQ, uint8_t* sK, uint8_t* sV, SharedBarriers& sb) {
+__device__ void attn_producer(const CUtensorMap* mapK, const CUtensorMap* mapV, const AttnParams& p, uint8_t* ring,
+                              SharedBarriers<AttnCfg<D, BN>::kRingK, AttnCfg<D, BN>::kRingV>& sb) {
   using C = AttnCfg<D, BN>;
+  constexpr int RK = C::kRingK, RV = C::kRingV;
+  uint8_t* k_ring = ring;
+  uint8_t* v_ring = ring + RK * C::kKVBytes;
   volatile int* abort = &sb.abort;
-  int g = 0, n = 0, bad = 0;
+  TileStream<BN, MODE> st;
+  st.start(p);
+  int jk = 0, jv = 0;
   bool ok = true;
-  for (int u = blockIdx.x; u < p.n_units && ok; u += gridDim.x) {
-    int b, h, qt;
-    decode_unit(p, u, b, h, qt);
-    const int kvh = h / p.group;
-    TileIter it = make_iter<BN, MODE>(p, b, kvh, qt);
-    int kb, bits;
-    if (!it.next(kb, bits)) {
-      bad |= it.bad;
-      continue;
-    }
-    const int qbuf = n & 1;
-    if (n >= 2 && !mbar_wait(&sb.q_empty[qbuf], ((n >> 1) - 1) & 1, abort)) {
+  auto load = [&](const CUtensorMap* map, uint8_t* base, uint64_t* full, uint64_t* empty, int R, int& j,
+                  const Tile& t) -> bool {
+    const int slot = j % R;
+    if (j >= R && !mbar_wait(&empty[slot], ((j / R) - 1) & 1, abort)) return false;
+    mbar_arrive_expect_tx(&full[slot], C::kKVBytes);
+    for (int i = 0; i < C::kBoxes; ++i)
+      tma_load_3d(base + slot * C::kKVBytes + i * BN * 128, map, &full[slot], 64 * i, t.kb * BN, t.z);
+    ++j;
+    return true;
+  };
+  Tile cur, nxt;
+  bool have = st.next(p, cur);
+  if (have && !load(mapK, k_ring, sb.k_full, sb.k_empty, RK, jk, cur)) ok = false;
+  while (have && ok) {
+    const bool more = st.next(p, nxt);
+    if (more && !load(mapK, k_ring, sb.k_full, sb.k_empty, RK, jk, nxt)) {
       ok = false;
       break;
     }
-    mbar_arrive_expect_tx(&sb.q_full[qbuf], C::kQBytes);
-    for (int i = 0; i < C::kBoxes; ++i)
-      tma_load_3d(sQ + qbuf * C::kQBytes + i * 128 * 128, mapQ, &sb.q_full[qbuf], 64 * i, qt * 128,
-                  b * p.n_heads + h);
-    ++n;
-    do {
-      const int s = g % C::kStages;
-      if (g >= C::kStages && !mbar_wait(&sb.kv_empty[s], ((g / C::kStages) - 1) & 1, abort)) {
-        ok = false;
-        break;
-      }
-      const int z = b * p.n_kv_heads + kvh;
-      mbar_arrive_expect_tx(&sb.k_full[s], C::kKVBytes);
-      for (int i = 0; i < C::kBoxes; ++i)
-        tma_load_3d(sK + s * C::kKVBytes + i * BN * 128, mapK, &sb.k_full[s], 64 * i, kb * BN, z);
-      mbar_arrive_expect_tx(&sb.v_full[s], C::kKVBytes);
-      for (int i = 0; i < C::kBoxes; ++i)
-        tma_load_3d(sV + s * C::kKVBytes + i * BN * 128, mapV, &sb.v_full[s], 64 * i, kb * BN, z);
-      ++g;
-    } while (it.next(kb, bits));
-    bad |= it.bad;
+    if (!load(mapV, v_ring, sb.v_full, sb.v_empty, RV, jv, cur)) {
+      ok = false;
+      break;
+    }
+    cur = nxt;
+    have = more;
   }
-  if (bad) atomicOr(p.status, kStatusBadSupport);
+  if (st.bad) atomicOr(p.status, kStatusBadSupport);
   if (!ok) {
-    raise_status(p, sb, kStatusTimeout);
+    raise_status(p, &sb.abort, kStatusTimeout);
     // Let every copy already issued land before the CTA's shared memory is
     // released.
     int never = 0;
-    for (int t = max(0, g - C::kStages); t < g; ++t) {
-      mbar_wait(&sb.k_full[t % C::kStages], (t / C::kStages) & 1, &never);
-      mbar_wait(&sb.v_full[t % C::kStages], (t / C::kStages) & 1, &never);
-    }
-    for (int m = max(0, n - 2); m < n; ++m) mbar_wait(&sb.q_full[m & 1], (m >> 1) & 1, &never);
+    for (int t = max(0, jk - RK); t < jk; ++t) mbar_wait(&sb.k_full[t % RK], (t / RK) & 1, &never);
+    for (int t = max(0, jv - RV); t < jv; ++t) mbar_wait(&sb.v_full[t % RV], (t / RV) & 1, &never);
   }
 }
 
-// ---------------------------------------------------------------- MMA issuer
-template <int D, int BN>
-__device__ __forceinline__ bool issue_pv(int t, bool first, uint32_t tmem, uint8_t* sP, uint8_t* sV,
-                                         SharedBarriers& sb) {
+// --------------------------------------------------------------- MMA issuers
+template <int D, int BN, int MODE>
+__device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* ring,
+                           SharedBarriers<AttnCfg<D, BN>::kRingK, AttnCfg<D, BN>::kRingV>& sb) {
   using C = AttnCfg<D, BN>;
+  constexpr int RK = C::kRingK;
   volatile int* abort = &sb.abort;
-  if (!mbar_wait(&sb.p_full, t & 1, abort)) return false;
-  const int s = t % C::kStages;
-  if (!mbar_wait(&sb.v_full[s], (t / C::kStages) & 1, abort)) return false;
-  tc_fence_after_sync();
-  constexpr uint32_t idesc = idesc_bf16_f32(128, D, false, true);
-  const uint32_t p_base = smem_u32(sP);
-  const uint32_t v_base = smem_u32(sV + s * C::kKVBytes);
-#pragma unroll
-  for (int kk = 0; kk < BN / 16; ++kk) {
-    const uint64_t a = smem_desc_sw128(p_base + (kk / 4) * 16384 + (kk % 4) * 32, 16, 1024);
-    const uint64_t bdesc = smem_desc_sw128(v_base + kk * 2048, BN * 128, 1024);
-    umma_bf16_ss(tmem + C::kTmemO, a, bdesc, idesc, (first && kk == 0) ? 0u : 1u);
+  constexpr uint32_t idesc_s = idesc_bf16_f32(128, BN, false, false);
+  TileStream<BN, MODE> st;
+  st.start(p);
+  int n_q = 0;
+  uint32_t q_col = 0;  // TMEM column of the current unit's Q
+  bool ok = true;
+  Tile t;
+  for (int j = 0; st.next(p, t); ++j) {
+    if (t.first) {
+      if (!mbar_wait(&sb.q_tmem, n_q & 1, abort)) ok = false;
+      q_col = C::kTmemQ + (n_q & 1) * C::kTmemQCols;
+      ++n_q;
+    }
+    const int slot = j % RK;
+    if (ok && !mbar_wait(&sb.k_full[slot], (j / RK) & 1, abort)) ok = false;
+    // S(j) overwrites the buffer that held P(j-2).
+    if (ok && j >= 2 && !mbar_wait(&sb.buf_free[j & 1], ((j >> 1) - 1) & 1, abort)) ok = false;
+    if (!ok) break;
+    tc_fence_after_sync();
+    const uint32_t s_col = C::kTmemS + (j & 1) * C::kTmemSCols;
+    const uint64_t b0 = smem_desc_sw128(smem_u32(ring + slot * C::kKVBytes), 16, 1024);
+#pragma unroll 1
+    for (int kk = 0; kk < D / 16; ++kk) {
+      // K step kk: 8 TMEM columns of Q; shared-memory descriptors of later
+      // steps differ only in the start address field (address >> 4).
+      const uint32_t b_off = ((kk >> 2) * (BN * 128) + (kk & 3) * 32) >> 4;
+      umma_bf16_ts(tmem + s_col, tmem + q_col + kk * 8, b0 + b_off, idesc_s, kk > 0 ? 1u : 0u);
+    }
+    umma_commit(&sb.s_full[j & 1]);
+    umma_commit(&sb.k_empty[slot]);
   }
-  umma_commit(&sb.kv_empty[s]);
-  umma_commit(&sb.o_full);
+  if (!ok) raise_status(p, &sb.abort, kStatusTimeout);
+  // Every MMA issued must have completed before TMEM is released.
+  umma_commit(&sb.s_done);
+  int never = 0;
+  mbar_wait(&sb.s_done, 0, &never);
+}
+
+template <int D, int BN, int MODE>
+__device__ void attn_mma_pv(const AttnParams& p, uint32_t tmem, uint8_t* ring,
+                            SharedBarriers<AttnCfg<D, BN>::kRingK, AttnCfg<D, BN>::kRingV>& sb) {
+  using C = AttnCfg<D, BN>;
+  constexpr int RK = C::kRingK, RV = C::kRingV;
+  uint8_t* v_ring = ring + RK * C::kKVBytes;
+  volatile int* abort = &sb.abort;
+  constexpr uint32_t idesc_o = idesc_bf16_f32(128, D, false, true);
+  TileStream<BN, MODE> st;
+  st.start(p);
+  bool ok = true;
+  Tile t;
+  for (int j = 0; st.next(p, t); ++j) {
+    const int slot = j % RV;
+    if (!mbar_wait(&sb.p_full, j & 1, abort)) ok = false;
+    if (ok && !mbar_wait(&sb.v_full[slot], (j / RV) & 1, abort)) ok = false;
+    if (!ok) break;
+    tc_fence_after_sync();
+    // P(j) sits in the first BN/2 columns of S buffer j & 1.
+    const uint32_t p_col = C::kTmemS + (j & 1) * C::kTmemSCols;
+    const uint64_t b0 = smem_desc_sw128(smem_u32(v_ring + slot * C::kKVBytes), BN * 128, 1024);
+#pragma unroll 1
+    for (int kk = 0; kk < BN / 16; ++kk)
+      umma_bf16_ts(tmem + C::kTmemO, tmem + p_col + kk * 8, b0 + ((kk * 2048) >> 4), idesc_o,
+                   (t.first && kk == 0) ? 0u : 1u);
+    umma_commit(&sb.o_full);
+    umma_commit(&sb.v_empty[slot]);
+    umma_commit(&sb.buf_free[j & 1]);
+  }
+  if (!ok) raise_status(p, &sb.abort, kStatusTimeout);
+  umma_commit(&sb.pv_done);
+  int never = 0;
+  mbar_wait(&sb.pv_done, 0, &never);
+}
+
+// Issues the TMA load of the Q tile of unit u into the staging buffer.
+template <int D, int BN>
+__device__ __forceinline__ void load_q(const CUtensorMap* mapQ, const AttnParams& p, int u, uint8_t* q_stage,
+                                       uint64_t* bar) {
+  using C = AttnCfg<D, BN>;
+  int b, h, qt;
+  decode_unit(p, u, b, h, qt);
+  mbar_arrive_expect_tx(bar, C::kQBytes);
+  for (int i = 0; i < C::kBoxes; ++i)
+    tma_load_3d(q_stage + i * 128 * 128, mapQ, bar, 64 * i, qt * 128, b * p.n_heads + h);
+}
+
+// First unit at or after u (stepping by stride) that has at least one tile.
+template <int BN, int MODE>
+__device__ __forceinline__ int next_nonempty_unit(const AttnParams& p, int u, int stride) {
+  for (; u < p.n_units; u += stride) {
+    if (MODE != kSparse) return u;
+    int b, h, qt;
+    decode_unit(p, u, b, h, qt);
+    auto it = make_iter<BN, MODE>(p, b, h / p.group, qt);
+    int kb, bits;
+    if (it.next(kb, bits)) return u;
+  }
+  return INT_MAX;
+}
+
+// Exchange of one float per row between the two softmax halves: thread
+// (half, row) publishes v and gets its partner's value.  Double-buffered by
+// phase; bounded wait.
+template <class SB>
+__device__ __forceinline__ bool half_exchange(SB& sb, int& phase, int half, int row, int lane,
+                                              float v, float& other, volatile int* abort) {
+  sb.xbuf[phase & 1][half][row] = v;
+  __syncwarp();
+  if (lane == 0) mbar_arrive(&sb.xch);
+  if (!warp_wait(&sb.xch, phase & 1, abort)) return false;
+  other = sb.xbuf[phase & 1][half ^ 1][row];
+  ++phase;
   return true;
 }
 
-template <int D, int BN, int MODE>
-__device__ void attn_mma(const AttnParams& p, uint32_t tmem, uint8_t* sQ, uint8_t* sK, uint8_t* sV, uint8_t* sP,
-                         SharedBarriers& sb) {
-  using C = AttnCfg<D, BN>;
-  volatile int* abort = &sb.abort;
-  constexpr uint32_t idesc_s = idesc_bf16_f32(128, BN, false, false);
-  int g = 0, n = 0;
-  bool ok = true;
-  for (int u = blockIdx.x; u < p.n_units && ok; u += gridDim.x) {
-    int b, h, qt;
-    decode_unit(p, u, b, h, qt);
-    TileIter it = make_iter<BN, MODE>(p, b, h / p.group, qt);
-    int kb, bits;
-    if (!it.next(kb, bits)) continue;
-    const int qbuf = n & 1;
-    if (!mbar_wait(&sb.q_full[qbuf], (n >> 1) & 1, abort)) {
-      ok = false;
-      break;
-    }
-    ++n;
-    const uint32_t q_base = smem_u32(sQ + qbuf * C::kQBytes);
-    int j = 0;
-    bool more;
-    do {
-      const int s = g % C::kStages;
-      if (!mbar_wait(&sb.k_full[s], (g / C::kStages) & 1, abort)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after_sync();
-      const uint32_t k_base = smem_u32(sK + s * C::kKVBytes);
-      const uint32_t s_tmem = tmem + (uint32_t)((g & 1) * BN);
-#pragma unroll
-      for (int kk = 0; kk < D / 16; ++kk) {
-        const uint64_t a = smem_desc_sw128(q_base + (kk / 4) * 16384 + (kk % 4) * 32, 16, 1024);
-        const uint64_t bdesc = smem_desc_sw128(k_base + (kk / 4) * (BN * 128) + (kk % 4) * 32, 16, 1024);
-        umma_bf16_ss(s_tmem, a, bdesc, idesc_s, kk > 0 ? 1u : 0u);
-      }
-      umma_commit(&sb.s_full[g & 1]);
-      more = it.next(kb, bits);
-      if (!more) umma_commit(&sb.q_empty[qbuf]);
-      if (j > 0 && !issue_pv<D, BN>(g - 1, j == 1, tmem, sP, sV, sb)) {
-        ok = false;
-        break;
-      }
-      ++g;
-      ++j;
-    } while (more);
-    if (ok && !issue_pv<D, BN>(g - 1, j == 1, tmem, sP, sV, sb)) ok = false;
-  }
-  if (!ok) raise_status(p, sb, kStatusTimeout);
-  // Every MMA issued must have completed before TMEM is released.
-  umma_commit(&sb.mma_done);
-  int never = 0;
-  mbar_wait(&sb.mma_done, 0, &never);
-}
-
 // ------------------------------------------------------------------- softmax
+// Warpgroup `half` of the softmax owns, for every query row of the tile,
+// key columns [half*BN/2, (half+1)*BN/2) of S and output columns
+// [half*D/2, (half+1)*D/2) of O.
 template <int D, int BN, int MODE>
-__device__ void attn_softmax(const AttnParams& p, uint32_t tmem, uint8_t* sP, SharedBarriers& sb) {
+__device__ void attn_softmax(const CUtensorMap* mapQ, const AttnParams& p, int half, uint32_t tmem,
+                             uint8_t* q_stage, SharedBarriers<AttnCfg<D, BN>::kRingK, AttnCfg<D, BN>::kRingV>& sb) {
   using C = AttnCfg<D, BN>;
+  constexpr int kCols = BN / 2;  // S columns per half
+  constexpr int kOCols = D / 2;  // O columns per half
   volatile int* abort = &sb.abort;
-  const int r = threadIdx.x;  // query row within the tile, 0..127
-  const int warp = r >> 5, lane = r & 31;
-  const uint32_t lane_tmem = tmem + ((uint32_t)(warp * 32) << 16);
-  const uint32_t p_base = smem_u32(sP);
+  const int r = threadIdx.x & 127;  // query row within the tile
+  const int wq = r >> 5, lane = r & 31;
+  const bool leader = (half == 0 && r == 0);
+  const uint32_t lane_tmem = tmem + ((uint32_t)(wq * 32) << 16);
   constexpr float kRescaleThreshold = 8.0f;  // log2 units: P stays <= 256
-  int g = 0, epi_phase = 0;
+  const int G = gridDim.x;
+  // Per-CTA scratch: [n_blocks][2][128] log2 partial masses, then
+  // [2][4][n_blocks] per-warp column sums.
+  float* scratch = p.scratch + (size_t)blockIdx.x * p.n_blocks * 264;
+  float* warp_sums = scratch + (size_t)p.n_blocks * 256;
+
+  // Q pipeline: the staging buffer holds the Q of unit q_next; copy_next()
+  // moves it into TMEM buffer n_q & 1 and prefetches the following one.
+  int q_next = next_nonempty_unit<BN, MODE>(p, blockIdx.x, G);
+  int n_q = 0, x_phase = 0, j = 0;
+  if (leader && q_next != INT_MAX) load_q<D, BN>(mapQ, p, q_next, q_stage, &sb.q_full);
   bool ok = true;
-  for (int u = blockIdx.x; u < p.n_units && ok; u += gridDim.x) {
+  auto copy_next = [&]() -> bool {
+    if (!warp_wait(&sb.q_full, n_q & 1, abort)) return false;
+    const uint32_t q_col = C::kTmemQ + (n_q & 1) * C::kTmemQCols;
+    if (half < C::kBoxes) {
+      const uint32_t box = smem_u32(q_stage + half * 128 * 128) + r * 128;
+      uint32_t w[32];
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {
+        const uint4 v = ld_shared_v4(box + ((c ^ (r & 7)) << 4));
+        w[4 * c + 0] = v.x;
+        w[4 * c + 1] = v.y;
+        w[4 * c + 2] = v.z;
+        w[4 * c + 3] = v.w;
+      }
+      tmem_st_32x32b_x32(lane_tmem + q_col + half * 32, w);
+      tmem_st_wait();
+    }
+    tc_fence_before_sync();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&sb.q_tmem);
+    const int following = next_nonempty_unit<BN, MODE>(p, q_next + G, G);
+    if (leader && following != INT_MAX) {
+      // Every warp has read the staging buffer once q_tmem completes.
+      if (!mbar_wait(&sb.q_tmem, n_q & 1, abort)) return false;
+      load_q<D, BN>(mapQ, p, following, q_stage, &sb.q_full);
+    }
+    q_next = following;
+    ++n_q;
+    return true;
+  };
+  if (q_next != INT_MAX && !copy_next()) ok = false;
+
+  for (int u = blockIdx.x; u < p.n_units && ok; u += G) {
     int b, h, qt;
     decode_unit(p, u, b, h, qt);
-    TileIter it = make_iter<BN, MODE>(p, b, h / p.group, qt);
+    auto it = make_iter<BN, MODE>(p, b, h / p.group, qt);
     const int row = qt * 128 + r;
     const int half_bit = (BN == 64) ? (1 << (r >> 6)) : 1;
     float m_ref = -INFINITY, l = 0.0f;
-    int j = 0, kb, bits, last_kb = -1;
-    while (it.next(kb, bits)) {
+    int jj = 0, kb, bits, last_kb = -1;
+    bool have = it.next(kb, bits);
+    // The next unit's Q goes into the other TMEM buffer while this one runs.
+    if (have && q_next != INT_MAX && !copy_next()) {
+      ok = false;
+      break;
+    }
+    while (have) {
+      int nkb, nbits;
+      const bool more = it.next(nkb, nbits);
       last_kb = kb;
-      const int sbuf = g & 1;
-      if (!warp_wait(&sb.s_full[sbuf], (g >> 1) & 1, abort)) {
+      const uint32_t s_col = C::kTmemS + (j & 1) * C::kTmemSCols;
+      if (!warp_wait(&sb.s_full[j & 1], (j >> 1) & 1, abort)) {
         ok = false;
         break;
       }
       tc_fence_after_sync();
-      float s[BN];
+      float s[kCols];
 #pragma unroll
-      for (int c = 0; c < BN / 32; ++c) {
+      for (int c = 0; c < kCols / 32; ++c) {
         uint32_t v[32];
-        tmem_ld_32x32b_x32(lane_tmem + sbuf * BN + 32 * c, v);
+        tmem_ld_32x32b_x32(lane_tmem + s_col + half * kCols + 32 * c, v);
         tmem_ld_wait(v);
 #pragma unroll
         for (int e = 0; e < 32; ++e) s[32 * c + e] = __uint_as_float(v[e]);
       }
-      const int k0 = kb * BN;
+      const int k0 = kb * BN + half * kCols;
       if (!(bits & half_bit)) {
 #pragma unroll
-        for (int c = 0; c < BN; ++c) s[c] = -INFINITY;
-      } else if (k0 + BN - 1 > row) {
+        for (int c = 0; c < kCols; ++c) s[c] = -INFINITY;
+      } else if (k0 + kCols - 1 > row) {
         const int lim = row - k0;  // keys k0 + c with c > lim are in the future
 #pragma unroll
-        for (int c = 0; c < BN; ++c) s[c] = (c > lim) ? -INFINITY : s[c];
+        for (int c = 0; c < kCols; ++c) s[c] = (c > lim) ? -INFINITY : s[c];
       }
       float mx8[8];
 #pragma unroll
       for (int e = 0; e < 8; ++e) mx8[e] = s[e];
 #pragma unroll
-      for (int c = 8; c < BN; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], s[c]);
-      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+      for (int c = 8; c < kCols; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], s[c]);
+      float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                       fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+      float mx_other;
+      if (!half_exchange(sb, x_phase, half, r, lane, mx, mx_other, abort)) {
+        ok = false;
+        break;
+      }
+      mx = fmaxf(mx, mx_other);
       const float m_tile = mx * p.scale_log2;
       float alpha = 1.0f;
       bool rescale = false;
@@ -404,175 +597,194 @@ __device__ void attn_softmax(const AttnParams& p, uint32_t tmem, uint8_t* sP, Sh
 #pragma unroll
       for (int e = 0; e < 8; ++e) sum8[e] = 0.0f;
 #pragma unroll
-      for (int c = 0; c < BN; ++c) {
+      for (int c = 0; c < kCols; ++c) {
         s[c] = ex2_approx(fmaf(s[c], p.scale_log2, -m_use));
         sum8[c & 7] += s[c];
       }
-      const float rowsum = ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) + ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
-      l += rowsum;
+      const float rowsum =
+          ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) + ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
+      l += rowsum;  // this half's part of the row sum
       if (MODE == kDenseMass)
-        p.scratch[((size_t)blockIdx.x * p.n_blocks + kb) * 128 + r] =
-            rowsum > 0.0f ? m_ref + lg2_approx(rowsum) : -INFINITY;
-      // The previous tile's P V must be complete before O is rescaled and the
-      // P buffer is overwritten.
-      if (g > 0) {
-        if (!warp_wait(&sb.o_full, (g - 1) & 1, abort)) {
+        scratch[((size_t)kb * 2 + half) * 128 + r] = rowsum > 0.0f ? m_ref + lg2_approx(rowsum) : -INFINITY;
+      // O is rescaled only after the previous P V completed.  tcgen05.ld/st
+      // are warp-collective: the warp rescales together, lanes whose max did
+      // not move use a factor of 1.
+      if (jj > 0 && __any_sync(0xffffffffu, rescale)) {
+        if (!warp_wait(&sb.o_full, (j - 1) & 1, abort)) {
           ok = false;
           break;
         }
         tc_fence_after_sync();
-      }
-      // tcgen05.ld/st are warp-collective: the warp rescales together, lanes
-      // whose max did not move use a factor of 1.
-      if (j > 0 && __any_sync(0xffffffffu, rescale)) {
         const float f = rescale ? alpha : 1.0f;
+        const uint32_t o_col = C::kTmemO + half * kOCols;
 #pragma unroll
-        for (int c = 0; c < D / 32; ++c) {
-          uint32_t v[32];
-          tmem_ld_32x32b_x32(lane_tmem + C::kTmemO + 32 * c, v);
+        for (int c = 0; c < kOCols / 16; ++c) {
+          uint32_t v[16];
+          tmem_ld_32x32b_x16(lane_tmem + o_col + 16 * c, v);
           tmem_ld_wait(v);
 #pragma unroll
-          for (int e = 0; e < 32; ++e) v[e] = __float_as_uint(__uint_as_float(v[e]) * f);
-          tmem_st_32x32b_x32(lane_tmem + C::kTmemO + 32 * c, v);
+          for (int e = 0; e < 16; ++e) v[e] = __float_as_uint(__uint_as_float(v[e]) * f);
+          tmem_st_32x32b_x16(lane_tmem + o_col + 16 * c, v);
         }
-        tmem_st_wait();
       }
+      // P as bf16 pairs: keys [half*kCols, (half+1)*kCols) of the row go to
+      // columns [half*kCols/2, (half+1)*kCols/2) of this tile's S buffer.
 #pragma unroll
-      for (int c8 = 0; c8 < BN / 8; ++c8) {
-        const uint32_t w0 = pack_bf16x2(s[8 * c8 + 0], s[8 * c8 + 1]);
-        const uint32_t w1 = pack_bf16x2(s[8 * c8 + 2], s[8 * c8 + 3]);
-        const uint32_t w2 = pack_bf16x2(s[8 * c8 + 4], s[8 * c8 + 5]);
-        const uint32_t w3 = pack_bf16x2(s[8 * c8 + 6], s[8 * c8 + 7]);
-        const uint32_t addr = p_base + (c8 / 8) * 16384 + r * 128 + (((c8 % 8) ^ (r & 7)) << 4);
-        st_shared_v4(addr, w0, w1, w2, w3);
+      for (int c = 0; c < kCols / 32; ++c) {
+        uint32_t w[16];
+#pragma unroll
+        for (int e = 0; e < 16; ++e) w[e] = pack_bf16x2(s[32 * c + 2 * e], s[32 * c + 2 * e + 1]);
+        tmem_st_32x32b_x16(lane_tmem + s_col + half * (kCols / 2) + 16 * c, w);
       }
-      fence_proxy_async_smem();
+      tmem_st_wait();
       tc_fence_before_sync();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sb.p_full);
-      ++g;
       ++j;
+      ++jj;
+      kb = nkb;
+      bits = nbits;
+      have = more;
     }
     if (!ok) break;
-    // ---- epilogue: O / l
-    if (j > 0) {
-      if (!warp_wait(&sb.o_full, (g - 1) & 1, abort)) {
+    // ---- epilogue: O / l over both halves
+    float l_other = 0.0f;
+    if (!half_exchange(sb, x_phase, half, r, lane, l, l_other, abort)) {
+      ok = false;
+      break;
+    }
+    const float l_row = half == 0 ? l + l_other : l_other + l;  // same order in both halves
+    if (jj > 0) {
+      if (!warp_wait(&sb.o_full, (j - 1) & 1, abort)) {
         ok = false;
         break;
       }
       tc_fence_after_sync();
     }
-    const float inv_l = l > 0.0f ? 1.0f / l : 0.0f;
-    __nv_bfloat16* orow = p.O + ((size_t)(b * p.n_heads + h) * p.seqlen + row) * D;
+    const float inv_l = l_row > 0.0f ? 1.0f / l_row : 0.0f;
+    __nv_bfloat16* orow = p.O + ((size_t)(b * p.n_heads + h) * p.seqlen + row) * D + half * kOCols;
 #pragma unroll
-    for (int c = 0; c < D / 32; ++c) {
-      uint32_t v[32];
-      if (j > 0) {
-        tmem_ld_32x32b_x32(lane_tmem + C::kTmemO + 32 * c, v);
+    for (int c = 0; c < kOCols / 16; ++c) {
+      uint32_t v[16];
+      if (jj > 0) {
+        tmem_ld_32x32b_x16(lane_tmem + C::kTmemO + half * kOCols + 16 * c, v);
         tmem_ld_wait(v);
       } else {
 #pragma unroll
-        for (int e = 0; e < 32; ++e) v[e] = 0u;
+        for (int e = 0; e < 16; ++e) v[e] = 0u;
       }
-      uint32_t w[16];
+      uint32_t w[8];
 #pragma unroll
-      for (int e = 0; e < 16; ++e)
+      for (int e = 0; e < 8; ++e)
         w[e] = pack_bf16x2(__uint_as_float(v[2 * e]) * inv_l, __uint_as_float(v[2 * e + 1]) * inv_l);
       if (row < p.seqlen) {
-        uint4* dst = reinterpret_cast<uint4*>(orow + 32 * c);
-#pragma unroll
-        for (int e = 0; e < 4; ++e) dst[e] = make_uint4(w[4 * e], w[4 * e + 1], w[4 * e + 2], w[4 * e + 3]);
+        uint4* dst = reinterpret_cast<uint4*>(orow + 16 * c);
+        dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
+        dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
       }
     }
     // ---- epilogue: block mass (Eq. 5)
     if (MODE == kDenseMass) {
-      float* red = reinterpret_cast<float*>(sP);  // every P V of this unit is complete
-      const float lse = m_ref + lg2_approx(l);
+      const float lse = m_ref + lg2_approx(l_row);
       const int n_kt = last_kb + 1;
       for (int t = 0; t < n_kt; ++t) {
-        const float lc = p.scratch[((size_t)blockIdx.x * p.n_blocks + t) * 128 + r];
+        const float lc = scratch[((size_t)t * 2 + half) * 128 + r];
         float v = (row < p.seqlen) ? ex2_approx(lc - lse) : 0.0f;
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-        if (lane == 0) red[warp * p.n_blocks + t] = v;
+        if (lane == 0) warp_sums[(half * 4 + wq) * p.n_blocks + t] = v;
       }
-      mbar_arrive(&sb.epi);
-      if (!warp_wait(&sb.epi, epi_phase & 1, abort)) {
+      // The exchange barrier orders the eight warps' global writes before
+      // the reads below (release/acquire at CTA scope).
+      float unused;
+      if (!half_exchange(sb, x_phase, half, r, lane, 0.0f, unused, abort)) {
         ok = false;
         break;
       }
-      ++epi_phase;
-      constexpr int kHalves = 128 / BN;
+      constexpr int kHalves = 128 / BN;  // query blocks per tile
       const float inv_b = 1.0f / (float)BN;
-      for (int e = r; e < kHalves * p.n_blocks; e += 128) {
+      const int tid = half * 128 + r;
+      for (int e = tid; e < kHalves * p.n_blocks; e += 256) {
         const int hf = e / p.n_blocks, t = e % p.n_blocks;
         const int qblock = qt * kHalves + hf;
         if (qblock >= p.n_blocks) continue;
         float* out = p.blockmass + ((size_t)(b * p.n_heads + h) * p.n_blocks + qblock) * p.n_blocks + t;
         if (t < n_kt) {
-          float sum;
-          if (BN == 128)
-            sum = (red[0 * p.n_blocks + t] + red[1 * p.n_blocks + t]) +
-                  (red[2 * p.n_blocks + t] + red[3 * p.n_blocks + t]);
-          else
-            sum = red[(2 * hf) * p.n_blocks + t] + red[(2 * hf + 1) * p.n_blocks + t];
+          float sum = 0.0f;
+          if (BN == 128) {
+#pragma unroll
+            for (int w = 0; w < 8; ++w) sum += warp_sums[w * p.n_blocks + t];
+          } else {
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh)
+#pragma unroll
+              for (int w = 2 * hf; w < 2 * hf + 2; ++w) sum += warp_sums[(hh * 4 + w) * p.n_blocks + t];
+          }
           sum *= inv_b;
           *out = (p.step == 0) ? sum : *out + sum;
         } else if (p.step == 0) {
           *out = 0.0f;
         }
       }
-      // `red` aliases the P tile, which the next unit overwrites.
-      mbar_arrive(&sb.epi);
-      if (!warp_wait(&sb.epi, epi_phase & 1, abort)) {
+      // warp_sums is rewritten by the next unit.
+      if (!half_exchange(sb, x_phase, half, r, lane, 0.0f, unused, abort)) {
         ok = false;
         break;
       }
-      ++epi_phase;
     }
   }
-  if (!ok) raise_status(p, sb, kStatusTimeout);
+  if (!ok) {
+    raise_status(p, &sb.abort, kStatusTimeout);
+    if (leader && n_q > 0) {
+      // Let a Q copy still in flight land before shared memory is released.
+      int never = 0;
+      mbar_wait(&sb.q_full, n_q & 1, &never);
+    }
+  }
 }
 
 // -------------------------------------------------------------------- kernel
 template <int D, int BN, int MODE>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(AttnCfg<D, BN>::kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
                 const __grid_constant__ CUtensorMap mapV, const AttnParams p) {
   using C = AttnCfg<D, BN>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* sQ = smem;
-  uint8_t* sK = sQ + 2 * C::kQBytes;
-  uint8_t* sV = sK + C::kStages * C::kKVBytes;
-  uint8_t* sP = sV + C::kStages * C::kKVBytes;
-  __shared__ SharedBarriers sb;
+  uint8_t* q_stage = smem;             // one Q tile
+  uint8_t* ring = smem + C::kQBytes;   // kRing K/V entries
+  __shared__ SharedBarriers<C::kRingK, C::kRingV> sb;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     sb.abort = 0;
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&sb.q_full[i], 1);
-      mbar_init(&sb.q_empty[i], 1);
-      mbar_init(&sb.s_full[i], 1);
-    }
-    for (int i = 0; i < C::kStages; ++i) {
+    for (int i = 0; i < C::kRingK; ++i) {
       mbar_init(&sb.k_full[i], 1);
-      mbar_init(&sb.v_full[i], 1);
-      mbar_init(&sb.kv_empty[i], 1);
+      mbar_init(&sb.k_empty[i], 1);
     }
-    mbar_init(&sb.p_full, 4);
+    for (int i = 0; i < C::kRingV; ++i) {
+      mbar_init(&sb.v_full[i], 1);
+      mbar_init(&sb.v_empty[i], 1);
+    }
+    mbar_init(&sb.q_full, 1);
+    mbar_init(&sb.q_tmem, 8);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&sb.s_full[b], 1);
+      mbar_init(&sb.buf_free[b], 1);
+    }
+    mbar_init(&sb.p_full, 8);
     mbar_init(&sb.o_full, 1);
-    mbar_init(&sb.mma_done, 1);
-    mbar_init(&sb.epi, 128);
+    mbar_init(&sb.xch, 8);
+    mbar_init(&sb.s_done, 1);
+    mbar_init(&sb.pv_done, 1);
     fence_mbar_init();
   }
-  if (warp == 4 && lane == 0) {
+  if (warp == C::kProducerWarp && lane == 0) {
     tma_prefetch_map(&mapQ);
     tma_prefetch_map(&mapK);
     tma_prefetch_map(&mapV);
   }
-  if (warp == 5) {
+  if (warp == C::kMmaSWarp) {
     tmem_alloc(&sb.tmem_base, C::kTmemCols);
     tmem_relinquish();
   }
@@ -581,18 +793,20 @@ __global__ void __launch_bounds__(192, 1)
   tc_fence_after_sync();
   const uint32_t tmem = sb.tmem_base;
 
-  if (warp < 4) {
-    attn_softmax<D, BN, MODE>(p, tmem, sP, sb);
-  } else if (warp == 4) {
-    if (lane == 0) attn_producer<D, BN, MODE>(&mapQ, &mapK, &mapV, p, sQ, sK, sV, sb);
-  } else {
-    if (lane == 0) attn_mma<D, BN, MODE>(p, tmem, sQ, sK, sV, sP, sb);
+  if (warp < 8) {
+    attn_softmax<D, BN, MODE>(&mapQ, p, warp >> 2, tmem, q_stage, sb);
+  } else if (warp == C::kProducerWarp) {
+    if (lane == 0) attn_producer<D, BN, MODE>(&mapK, &mapV, p, ring, sb);
+  } else if (warp == C::kMmaSWarp) {
+    if (lane == 0) attn_mma_s<D, BN, MODE>(p, tmem, ring, sb);
+  } else if (warp == C::kMmaPVWarp) {
+    if (lane == 0) attn_mma_pv<D, BN, MODE>(p, tmem, ring, sb);
   }
 
   __syncwarp();
   tc_fence_before_sync();
   __syncthreads();
-  if (warp == 5) {
+  if (warp == C::kMmaSWarp) {
     __syncwarp();
     tc_fence_after_sync();
     tmem_dealloc(tmem, C::kTmemCols);

@@ -28,7 +28,8 @@ struct AttnParams {
   const int32_t* idx;     // kSparse
   const int32_t* counts;  // kSparse
   int cap;                // kSparse
-  float* scratch;         // kDenseMass: [gridDim.x][n_blocks][128] log2 partial masses
+  float* scratch;         // kDenseMass: per CTA [n_blocks][2][128] log2 partial masses followed
+                          // by [2][4][n_blocks] per-warp sums
   int* status;
 };
 

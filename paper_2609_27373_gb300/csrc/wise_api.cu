@@ -136,8 +136,6 @@ int launch_attention(const wise_shape_t* sh, const void* Q, const void* K, const
   const int n_blocks = sh->seqlen / sh->block;
   if (mode == kDenseMass) {
     if (!aligned(blockmass, 4) || step < 0) return WISE_ERR_INVALID_ARG;
-    // The epilogue's cross-warp reduction reuses the P tile: 4 * nKB floats.
-    if (4 * n_blocks * 4 > (sh->block / 64) * 128 * 128) return WISE_ERR_UNSUPPORTED;
   }
   if (mode == kSparse) {
     if (!idx || !counts || !aligned(idx, 4) || !aligned(counts, 4) || cap <= 0) return WISE_ERR_INVALID_ARG;
@@ -178,7 +176,9 @@ int launch_attention(const wise_shape_t* sh, const void* Q, const void* K, const
   L.stream = stream;
   p.scratch = nullptr;
   if (mode == kDenseMass) {
-    const size_t need = (size_t)L.grid * n_blocks * 128 * sizeof(float);
+    // Per CTA: [nKB][2][128] log2 partial masses and [2][4][nKB] per-warp
+    // sums.
+    const size_t need = (size_t)L.grid * n_blocks * 264 * sizeof(float);
     if (caller_scratch) {
       if (need > caller_scratch_bytes) return WISE_ERR_UNSUPPORTED;
       p.scratch = caller_scratch;
