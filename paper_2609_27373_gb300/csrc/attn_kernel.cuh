@@ -59,6 +59,12 @@
 #include "internal.cuh"
 #include "ptx.cuh"
 
+// Pairs (of every 8) of softmax exponentials evaluated on the FMA pipe
+// instead of MUFU (0 = all on MUFU).
+#ifndef WISE_EMU_PAIRS
+#define WISE_EMU_PAIRS 0
+#endif
+
 namespace wise {
 
 template <int D, int BN>
@@ -101,6 +107,85 @@ __device__ __forceinline__ float lg2_approx(float x) {
   float y;
   asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// Maximum of n values with a tree of three-input max operations.
+template <int N>
+__device__ __forceinline__ float row_max(const float (&s)[N]) {
+  float m[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) m[e] = s[e];
+#pragma unroll
+  for (int c = 8; c + 1 < N; c += 16) {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) m[e] = fmax3(m[e], s[c + e], (c + 8 + e < N) ? s[c + 8 + e] : s[c + e]);
+  }
+  return fmaxf(fmax3(m[0], m[1], m[2]), fmax3(fmax3(m[3], m[4], m[5]), m[6], m[7]));
+}
+
+// 2^x for a pair of values on the FMA and integer pipes, leaving the MUFU
+// unit to the other exponentials (the softmax is otherwise bound by MUFU
+// throughput, 16 ex2 per clock per SM).  Cody-Waite style reduction: adding
+// 1.5 * 2^23 rounds x to the nearest integer n (which also appears in the low
+// mantissa bits of the sum), f = x - n lies in [-1/2, 1/2], 2^f is a degree-3
+// polynomial fitted here to minimise the maximum relative error on that
+// interval (7.5e-5 with fp32 Horner evaluation), and n is added to the
+// exponent field.  Inputs are clamped to [-126, 64] (so the exponent field
+// cannot wrap); the results feed bf16 probabilities (relative precision
+// 3.9e-3).  Masked inputs (-inf) need exp2_scaled's masked path for an exact 0.
+__device__ __forceinline__ float2 exp2_poly2(float2 x) {
+  constexpr float kRound = 12582912.0f;  // 1.5 * 2^23
+  const float2 xc = make_float2(fminf(fmaxf(x.x, -126.0f), 64.0f), fminf(fmaxf(x.y, -126.0f), 64.0f));
+  const float2 t = __fadd2_rn(xc, make_float2(kRound, kRound));
+  const float2 n = __fadd2_rn(t, make_float2(-kRound, -kRound));
+  const float2 f = __fadd2_rn(xc, make_float2(-n.x, -n.y));
+  float2 q = __ffma2_rn(make_float2(5.517166853e-02f, 5.517166853e-02f), f,
+                        make_float2(2.426111251e-01f, 2.426111251e-01f));
+  q = __ffma2_rn(q, f, make_float2(6.932609677e-01f, 6.932609677e-01f));
+  q = __ffma2_rn(q, f, make_float2(9.999280572e-01f, 9.999280572e-01f));
+  // The rounded integer sits in the low mantissa bits of t: shift it into the
+  // exponent field (the constant part of t's bits cancels modulo 2^32).
+  constexpr int kBias = (int)(0x4B400000u << 23);
+  return make_float2(__int_as_float(__float_as_int(q.x) + (__float_as_int(t.x) << 23) - kBias),
+                     __int_as_float(__float_as_int(q.y) + (__float_as_int(t.y) << 23) - kBias));
+}
+
+// p = 2^(s * scale - shift) in place, two elements per packed FMA; returns
+// the sum of p.  kEmu of every 8 pairs use exp2_poly2, the rest MUFU ex2.
+// With `masked` (the row has masked keys in this tile) emulated results of
+// inputs below -126 are forced to exactly 0, as ex2 gives for -inf.
+template <int kEmu, int N>
+__device__ __forceinline__ float exp2_scaled(float (&s)[N], float scale, float shift, bool masked) {
+  const float2 sc = make_float2(scale, scale), sh = make_float2(-shift, -shift);
+  float2 acc[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) acc[e] = make_float2(0.0f, 0.0f);
+#pragma unroll
+  for (int c = 0; c < N; c += 2) {
+    const float2 x = __ffma2_rn(make_float2(s[c], s[c + 1]), sc, sh);
+    float2 y;
+    if ((c / 2) % 8 < kEmu) {
+      y = exp2_poly2(x);
+      if (masked) {
+        y.x = x.x < -126.0f ? 0.0f : y.x;
+        y.y = x.y < -126.0f ? 0.0f : y.y;
+      }
+    } else {
+      y.x = ex2_approx(x.x);
+      y.y = ex2_approx(x.y);
+    }
+    s[c] = y.x;
+    s[c + 1] = y.y;
+    acc[(c / 2) & 3] = __fadd2_rn(acc[(c / 2) & 3], y);
+  }
+  const float2 b = __fadd2_rn(__fadd2_rn(acc[0], acc[1]), __fadd2_rn(acc[2], acc[3]));
+  return b.x + b.y;
 }
 
 // Key tiles of one unit in ascending order.  Dense: 0..last.  Sparse: the
@@ -273,11 +358,15 @@ struct TileStream {
 template <int RK, int RV>
 struct SharedBarriers {
   uint64_t k_full[RK], k_empty[RK], v_full[RV], v_empty[RV];
+  // Barriers that a thread may reach late (after the producing side has
+  // already moved on by one item) exist once per buffer: a second completion
+  // of the same barrier then needs work that the waiting thread itself has
+  // not issued yet, so a parity wait can never skip a phase.
   uint64_t q_full;       // Q tile landed in the staging buffer (TMA)
-  uint64_t q_tmem;       // Q tile copied into TMEM (8 softmax warps)
+  uint64_t q_tmem[2];    // Q copied into TMEM buffer b (8 softmax warps)
   uint64_t s_full[2];    // S buffer b written (S thread commit)
   uint64_t buf_free[2];  // P of buffer b consumed by its P V (P V thread commit)
-  uint64_t p_full;       // P written into TMEM (8 softmax warps)
+  uint64_t p_full[2];    // P of buffer b written into TMEM (8 softmax warps)
   uint64_t o_full;       // a P V completed (P V thread commit)
   uint64_t xch;          // the two softmax halves exchanged row values (8 warps)
   uint64_t s_done, pv_done;
@@ -363,7 +452,7 @@ __device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* ring,
   Tile t;
   for (int j = 0; st.next(p, t); ++j) {
     if (t.first) {
-      if (!mbar_wait(&sb.q_tmem, n_q & 1, abort)) ok = false;
+      if (!mbar_wait(&sb.q_tmem[n_q & 1], (n_q >> 1) & 1, abort)) ok = false;
       q_col = C::kTmemQ + (n_q & 1) * C::kTmemQCols;
       ++n_q;
     }
@@ -406,7 +495,7 @@ __device__ void attn_mma_pv(const AttnParams& p, uint32_t tmem, uint8_t* ring,
   Tile t;
   for (int j = 0; st.next(p, t); ++j) {
     const int slot = j % RV;
-    if (!mbar_wait(&sb.p_full, j & 1, abort)) ok = false;
+    if (!mbar_wait(&sb.p_full[j & 1], (j >> 1) & 1, abort)) ok = false;
     if (ok && !mbar_wait(&sb.v_full[slot], (j / RV) & 1, abort)) ok = false;
     if (!ok) break;
     tc_fence_after_sync();
@@ -453,19 +542,58 @@ __device__ __forceinline__ int next_nonempty_unit(const AttnParams& p, int u, in
   return INT_MAX;
 }
 
+// Loads this thread's kCols columns of an S tile (one or two 32-column
+// loads, one wait) and applies the causal / support masks.
+template <int kCols>
+__device__ __forceinline__ void load_s_half(uint32_t addr, float (&s)[kCols], bool attend, int lim) {
+  uint32_t va[32], vb[32];
+  tmem_ld_32x32b_x32(addr, va);
+  if constexpr (kCols == 64) {
+    tmem_ld_32x32b_x32(addr + 32, vb);
+    tmem_ld_wait(va, vb);
+  } else {
+    tmem_ld_wait(va);
+  }
+#pragma unroll
+  for (int e = 0; e < 32; ++e) s[e] = __uint_as_float(va[e]);
+  if constexpr (kCols == 64) {
+#pragma unroll
+    for (int e = 0; e < 32; ++e) s[32 + e] = __uint_as_float(vb[e]);
+  }
+  if (!attend) {
+#pragma unroll
+    for (int c = 0; c < kCols; ++c) s[c] = -INFINITY;
+  } else if (lim < kCols - 1) {
+    // keys with column c > lim are in the future of this row
+#pragma unroll
+    for (int c = 0; c < kCols; ++c) s[c] = (c > lim) ? -INFINITY : s[c];
+  }
+}
+
 // Exchange of one float per row between the two softmax halves: thread
 // (half, row) publishes v and gets its partner's value.  Double-buffered by
 // phase; bounded wait.
 template <class SB>
-__device__ __forceinline__ bool half_exchange(SB& sb, int& phase, int half, int row, int lane,
-                                              float v, float& other, volatile int* abort) {
+__device__ __forceinline__ void half_publish(SB& sb, int phase, int half, int row, int lane, float v) {
   sb.xbuf[phase & 1][half][row] = v;
   __syncwarp();
   if (lane == 0) mbar_arrive(&sb.xch);
+}
+
+template <class SB>
+__device__ __forceinline__ bool half_collect(SB& sb, int& phase, int half, int row, float& other,
+                                             volatile int* abort) {
   if (!warp_wait(&sb.xch, phase & 1, abort)) return false;
   other = sb.xbuf[phase & 1][half ^ 1][row];
   ++phase;
   return true;
+}
+
+template <class SB>
+__device__ __forceinline__ bool half_exchange(SB& sb, int& phase, int half, int row, int lane,
+                                              float v, float& other, volatile int* abort) {
+  half_publish(sb, phase, half, row, lane, v);
+  return half_collect(sb, phase, half, row, other, abort);
 }
 
 // ------------------------------------------------------------------- softmax
@@ -478,6 +606,9 @@ __device__ void attn_softmax(const CUtensorMap* mapQ, const AttnParams& p, int h
   using C = AttnCfg<D, BN>;
   constexpr int kCols = BN / 2;  // S columns per half
   constexpr int kOCols = D / 2;  // O columns per half
+  // Pairs of every 8 whose exponential runs on the FMA pipe; the block-mass
+  // variant keeps the hardware ex2 throughout for its sums.
+  constexpr int kEmu = (MODE == kDenseMass) ? 0 : WISE_EMU_PAIRS;
   volatile int* abort = &sb.abort;
   const int r = threadIdx.x & 127;  // query row within the tile
   const int wq = r >> 5, lane = r & 31;
@@ -515,11 +646,11 @@ __device__ void attn_softmax(const CUtensorMap* mapQ, const AttnParams& p, int h
     }
     tc_fence_before_sync();
     __syncwarp();
-    if (lane == 0) mbar_arrive(&sb.q_tmem);
+    if (lane == 0) mbar_arrive(&sb.q_tmem[n_q & 1]);
     const int following = next_nonempty_unit<BN, MODE>(p, q_next + G, G);
     if (leader && following != INT_MAX) {
       // Every warp has read the staging buffer once q_tmem completes.
-      if (!mbar_wait(&sb.q_tmem, n_q & 1, abort)) return false;
+      if (!mbar_wait(&sb.q_tmem[n_q & 1], (n_q >> 1) & 1, abort)) return false;
       load_q<D, BN>(mapQ, p, following, q_stage, &sb.q_full);
     }
     q_next = following;
@@ -552,38 +683,29 @@ __device__ void attn_softmax(const CUtensorMap* mapQ, const AttnParams& p, int h
         break;
       }
       tc_fence_after_sync();
-      float s[kCols];
-#pragma unroll
-      for (int c = 0; c < kCols / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld_32x32b_x32(lane_tmem + s_col + half * kCols + 32 * c, v);
-        tmem_ld_wait(v);
-#pragma unroll
-        for (int e = 0; e < 32; ++e) s[32 * c + e] = __uint_as_float(v[e]);
-      }
       const int k0 = kb * BN + half * kCols;
-      if (!(bits & half_bit)) {
-#pragma unroll
-        for (int c = 0; c < kCols; ++c) s[c] = -INFINITY;
-      } else if (k0 + kCols - 1 > row) {
-        const int lim = row - k0;  // keys k0 + c with c > lim are in the future
-#pragma unroll
-        for (int c = 0; c < kCols; ++c) s[c] = (c > lim) ? -INFINITY : s[c];
-      }
-      float mx8[8];
-#pragma unroll
-      for (int e = 0; e < 8; ++e) mx8[e] = s[e];
-#pragma unroll
-      for (int c = 8; c < kCols; ++c) mx8[c & 7] = fmaxf(mx8[c & 7], s[c]);
-      float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                       fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+      const bool attend = (bits & half_bit) != 0;
+      const int lim = row - k0;  // keys k0 + c with c > lim are in the future
+      const uint32_t s_addr = lane_tmem + s_col + half * kCols;
+      float s[kCols];
+      load_s_half<kCols>(s_addr, s, attend, lim);
+      const float mx_local = row_max(s);
+      // The partner half's maximum is needed before the exponentials can be
+      // trusted; publish now and collect after them.  Past a unit's first
+      // tile the running max rarely moves, so the exponentials are computed
+      // speculatively against it and redone only where it did move.
+      half_publish(sb, x_phase, half, r, lane, mx_local);
+      const bool first_tile = (jj == 0);
+      const float m_old = m_ref;
+      float rowsum = 0.0f;
+      const bool masked = !attend || lim < kCols - 1;
+      if (!first_tile) rowsum = exp2_scaled<kEmu>(s, p.scale_log2, m_old == -INFINITY ? 0.0f : m_old, masked);
       float mx_other;
-      if (!half_exchange(sb, x_phase, half, r, lane, mx, mx_other, abort)) {
+      if (!half_collect(sb, x_phase, half, r, mx_other, abort)) {
         ok = false;
         break;
       }
-      mx = fmaxf(mx, mx_other);
-      const float m_tile = mx * p.scale_log2;
+      const float m_tile = fmaxf(mx_local, mx_other) * p.scale_log2;
       float alpha = 1.0f;
       bool rescale = false;
       if (m_tile > m_ref + kRescaleThreshold) {
@@ -593,16 +715,29 @@ __device__ void attn_softmax(const CUtensorMap* mapQ, const AttnParams& p, int h
         l *= alpha;
       }
       const float m_use = (m_ref == -INFINITY) ? 0.0f : m_ref;
-      float sum8[8];
+      if (first_tile) {
+        rowsum = exp2_scaled<kEmu>(s, p.scale_log2, m_use, masked);
+      } else if (__any_sync(0xffffffffu, m_ref != m_old)) {
+        // Redo the rows whose running max moved (S is still in TMEM).
+        float t[kCols];
+        load_s_half<kCols>(s_addr, t, attend, lim);
+        const float tsum = exp2_scaled<kEmu>(t, p.scale_log2, m_use, masked);
+        if (m_ref != m_old) {
+          rowsum = tsum;
 #pragma unroll
-      for (int e = 0; e < 8; ++e) sum8[e] = 0.0f;
-#pragma unroll
-      for (int c = 0; c < kCols; ++c) {
-        s[c] = ex2_approx(fmaf(s[c], p.scale_log2, -m_use));
-        sum8[c & 7] += s[c];
+          for (int c = 0; c < kCols; ++c) s[c] = t[c];
+        }
       }
-      const float rowsum =
-          ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) + ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
+      // P as bf16 pairs: keys [half*kCols, (half+1)*kCols) of the row go to
+      // columns [half*kCols/2, (half+1)*kCols/2) of this tile's S buffer.
+      // The stores complete while the bookkeeping below runs.
+#pragma unroll
+      for (int c = 0; c < kCols / 32; ++c) {
+        uint32_t w[16];
+#pragma unroll
+        for (int e = 0; e < 16; ++e) w[e] = pack_bf16x2(s[32 * c + 2 * e], s[32 * c + 2 * e + 1]);
+        tmem_st_32x32b_x16(lane_tmem + s_col + half * (kCols / 2) + 16 * c, w);
+      }
       l += rowsum;  // this half's part of the row sum
       if (MODE == kDenseMass)
         scratch[((size_t)kb * 2 + half) * 128 + r] = rowsum > 0.0f ? m_ref + lg2_approx(rowsum) : -INFINITY;
@@ -627,19 +762,10 @@ __device__ void attn_softmax(const CUtensorMap* mapQ, const AttnParams& p, int h
           tmem_st_32x32b_x16(lane_tmem + o_col + 16 * c, v);
         }
       }
-      // P as bf16 pairs: keys [half*kCols, (half+1)*kCols) of the row go to
-      // columns [half*kCols/2, (half+1)*kCols/2) of this tile's S buffer.
-#pragma unroll
-      for (int c = 0; c < kCols / 32; ++c) {
-        uint32_t w[16];
-#pragma unroll
-        for (int e = 0; e < 16; ++e) w[e] = pack_bf16x2(s[32 * c + 2 * e], s[32 * c + 2 * e + 1]);
-        tmem_st_32x32b_x16(lane_tmem + s_col + half * (kCols / 2) + 16 * c, w);
-      }
       tmem_st_wait();
       tc_fence_before_sync();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&sb.p_full);
+      if (lane == 0) mbar_arrive(&sb.p_full[j & 1]);
       ++j;
       ++jj;
       kb = nkb;
@@ -767,12 +893,12 @@ __global__ void __launch_bounds__(AttnCfg<D, BN>::kThreads, 1)
       mbar_init(&sb.v_empty[i], 1);
     }
     mbar_init(&sb.q_full, 1);
-    mbar_init(&sb.q_tmem, 8);
     for (int b = 0; b < 2; ++b) {
+      mbar_init(&sb.q_tmem[b], 8);
       mbar_init(&sb.s_full[b], 1);
       mbar_init(&sb.buf_free[b], 1);
+      mbar_init(&sb.p_full[b], 8);
     }
-    mbar_init(&sb.p_full, 8);
     mbar_init(&sb.o_full, 1);
     mbar_init(&sb.xch, 8);
     mbar_init(&sb.s_done, 1);
