@@ -118,9 +118,10 @@ int wise_full_attn_accumulate(const wise_shape_t* shape, const void* Q, const vo
  * Arguments, layouts and results are those of wise_full_attn_accumulate;
  * blockmass must not be NULL (plain dense attention uses no scratch).
  * Limit: one call needs min(batch*n_heads*ceil(seqlen/128), SM count) *
- * nKB * 1056 bytes of scratch; larger problems return WISE_ERR_UNSUPPORTED and
- * launch nothing.  On a 152-SM GB300 with at least 152 query tiles that is
- * nKB <= 52 (seqlen <= 6656 with block 128).
+ * (2048 * (nKB/2 + 1) + 64 * nKB) bytes of scratch (nKB/2 rounded down);
+ * larger problems return WISE_ERR_UNSUPPORTED and launch nothing.  On a
+ * 152-SM GB300 with at least 152 query tiles that is nKB <= 49 (seqlen <=
+ * 6272 with block 128).
  * The first call on each device looks up the array's device address (with
  * that device current) and caches it; make that first call before any CUDA
  * stream capture.  All calls on a device share the one array: calls whose

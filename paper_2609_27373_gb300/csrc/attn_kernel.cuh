@@ -5,65 +5,71 @@
 //   kSparse     key blocks restricted to the selected support      (Eqs. 7-8)
 //
 // Work decomposition.  A unit is one 128-row query tile of one (batch, head);
-// units are numbered in order of decreasing causal length, and the
-// persistent grid (one CTA per SM) hands CTA c the units c, c + grid, ...
-// Each unit walks its list of key tiles (BN = block keys each): every tile of
-// the causal prefix (dense), or the blocks of the support (sparse; with block
-// 64 a query tile covers two query blocks and walks the union of their lists,
-// masking per half).
+// units are numbered in order of decreasing causal length.  The persistent
+// grid (one CTA per SM) deals them out in a snake order (CTA c takes unit
+// k*G + c in even rounds k and k*G + G-1-c in odd rounds), which evens out
+// the per-CTA sums of the decreasing lengths.  Each unit walks its list of
+// key tiles (BN keys each): every tile of the causal prefix (dense), or the
+// blocks of the support (sparse; with block 64 a query tile covers two query
+// blocks and walks the union of their lists, masking per half).
 //
 // Both products run with the A operand in tensor memory, because a tcgen05
 // MMA that reads both operands from shared memory is limited by the shared
 // memory read rate to about half the tensor peak (measured: 118 clk per
 // M128/N128/K16 step with both operands in shared memory, 66 clk with A in
 // TMEM):
-//   S = Q K^T    Q copied once per unit from shared memory into TMEM, K
-//                from shared memory (K-major);
+//   S = Q K^T    Q copied per unit from shared memory into TMEM with
+//                tcgen05.cp (ordered before the MMAs that read it), K from
+//                shared memory (K-major);
 //   O += P V     P written by the softmax into TMEM, V from shared memory
 //                (MN-major).
 // TMEM (512 columns): Q double-buffered across units (2 x 64 columns), S
 // double-buffered across tiles (2 x 128 columns, P overwrites the first BN/2
 // columns of its S), O (128 columns).
 //
-// Warp roles (352 threads):
-//   warps 0-3 and 4-7  two softmax warpgroups.  Thread t of warpgroup h owns
-//              query row t (= TMEM lane t), key columns [h BN/2, (h+1) BN/2)
-//              of every S tile and output columns [h D/2, (h+1) D/2) of O.
-//              Per tile it loads its half row of S, exchanges the half-row
-//              maximum with its partner thread (bounded mbarrier), keeps the
-//              running max and its half of the row sum (online softmax in the
-//              log2 domain; O is rescaled only when the max grows by more than
-//              2^8), and writes its half of P into TMEM.  Per unit it copies
-//              the next unit's Q into TMEM and runs the epilogue: O / l to
-//              global memory and, for kDenseMass, the block masses.
-//   warp 8     TMA producer: K tiles into a ring of kRingK entries and V tiles
-//              into a ring of kRingV entries, in the order K(0), K(1), V(0),
-//              K(2), V(1), ...
-//   warp 9     S issuer: S(j) = Q K(j)^T into S buffer j & 1, one tile ahead
-//              of the softmax.
+// Warp roles (384 threads; warp 11 only completes warpgroup 2):
+//   warp 8     producer.  Walks the CTA's units, validates the support lists,
+//              and publishes the tile schedule (one entry per tile, plus
+//              markers for units without tiles and for the end) in a
+//              shared-memory ring that every other role reads; issues the
+//              TMA loads of Q (staging buffer), K (ring of kRingK) and V (ring
+//              of kRingV) in the order Q, K(0), K(1), V(0), K(2), V(1), ...
+//   warp 9     S issuer: copies each unit's Q into TMEM and issues
+//              S(j) = Q K(j)^T into S buffer j & 1.
 //   warp 10    P V issuer: O += P(j) V(j) once the softmax has written P(j).
-//   A tcgen05.mma issue blocks its thread while the tensor core drains the
-//   previous instructions, so the two products are issued from two threads:
-//   each thread's barrier checks overlap the other's issue and the tensor
-//   core stays fed.  S(j) reuses the buffer of P(j-2); the P V thread commits
-//   buf_free[b] after each P V so that the S thread can wait for it.
+//              A tcgen05.mma issue blocks its thread while the tensor core
+//              drains earlier instructions, so the two products are issued
+//              from two threads.
+//   warps 0-3 and 4-7  softmax warpgroups 0 and 1.  Warpgroup w handles the
+//              tiles j with j & 1 == w (so it always uses S buffer w); thread
+//              t of a warpgroup owns query row t (= TMEM lane t) and the whole
+//              row of each of its tiles.  The online softmax runs in the log2
+//              domain with one running max m per row shared by both
+//              warpgroups: for tile j, the handler needs m after tile j-1
+//              (from the other warpgroup, through shared memory) and
+//              publishes m after tile j; O is rescaled only when m grows by
+//              more than 2^8.  Each warpgroup keeps its own part of the row
+//              sum; the two parts are combined at the end of the unit.  Since
+//              the two warpgroups work on different tiles, one computes
+//              exponentials while the other loads S or writes P.
+//   Epilogue.  O / l goes to global memory in two column halves, one per
+//              warpgroup.  The warpgroup that handled the unit's last tile
+//              writes its half at once; the other one first runs its tile of
+//              the next unit (its next tile always is that unit's first) and
+//              then writes its half, so that the tensor core receives the
+//              next P while the epilogue runs.  The first P V of a unit waits
+//              until both halves have read O.
 //
+// Every wait is bounded (kWaitLimitNs); a wait that runs out sets the status
+// word and an abort flag, and every role unwinds.
 #pragma once
 
 #include <cuda_bf16.h>
 #include <limits.h>
 #include <stdint.h>
 
-#include <type_traits>
-
 #include "internal.cuh"
 #include "ptx.cuh"
-
-// Pairs (of every 8) of softmax exponentials evaluated on the FMA pipe
-// instead of MUFU (0 = all on MUFU).
-#ifndef WISE_EMU_PAIRS
-#define WISE_EMU_PAIRS 0
-#endif
 
 namespace wise {
 
@@ -72,9 +78,10 @@ struct AttnCfg {
   static constexpr int kBoxes = (D + 63) / 64;          // 64-column TMA boxes per row tile
   static constexpr int kQBytes = kBoxes * 128 * 128;    // one 128-row Q tile (staging)
   static constexpr int kKVBytes = kBoxes * BN * 128;    // one BN-row K or V tile (one ring entry)
-  // Dynamic shared memory available after the 1024-byte alignment slack and
-  // the static barriers and exchange buffers.
-  static constexpr int kBudget = 227 * 1024 - 1024 - 2560;
+  // Static shared memory (barriers, schedule ring, row exchange buffers).
+  static constexpr int kStaticReserve = 6 * 1024;
+  // Dynamic shared memory available after the 1024-byte alignment slack.
+  static constexpr int kBudget = 227 * 1024 - 1024 - kStaticReserve;
   static constexpr int kRingFit = (kBudget - kQBytes) / kKVBytes;
   static constexpr int kRing = kRingFit > 12 ? 12 : kRingFit;
   static constexpr int kRingK = (kRing + 1) / 2;  // K tiles (consumed by S)
@@ -89,13 +96,29 @@ struct AttnCfg {
   static constexpr uint32_t kTmemSCols = 128;
   static constexpr uint32_t kTmemO = 384;     // O accumulator
   static constexpr uint32_t kTmemCols = 512;
-  static constexpr int kThreads = 352;
+  // Warps 0-7 softmax, 8 producer, 9 and 10 MMA issuers, 11 idle (it
+  // completes warpgroup 2 for setmaxnreg).  Launch: 384 x 168 registers;
+  // after the split 256 x kRegsSoftmax + 128 x kRegsOther = 64512.
+  static constexpr int kThreads = 384;
+  static constexpr int kRegsSoftmax = 224;
+  static constexpr int kRegsOther = 56;
   static constexpr int kProducerWarp = 8;
   static constexpr int kMmaSWarp = 9;   // issues S = Q K^T, owns the TMEM allocation
   static constexpr int kMmaPVWarp = 10; // issues O += P V
   static_assert(kRingV >= 1 && kRingK >= 2, "shared memory budget");
   static_assert(BN <= 128 && D <= 128, "TMEM budget");
+  static_assert(256 * kRegsSoftmax + 128 * kRegsOther <= kThreads * 168, "register split");
 };
+
+// Tile schedule ring.  Entry = {key block, unit, flags, 0}; the low two flag
+// bits say which 64-row halves of the query tile attend the key block.
+constexpr int kSchedSlots = 32;
+constexpr int kEntFirst = 4;   // first tile of its unit
+constexpr int kEntLast = 8;    // last tile of its unit
+constexpr int kEntEmpty = 16;  // unit without tiles (its output rows are zero)
+constexpr int kEntEnd = 32;    // no more units for this CTA
+// Readers of every entry: the two MMA threads and the eight softmax warps.
+constexpr int kSchedReaders = 10;
 
 __device__ __forceinline__ float ex2_approx(float x) {
   float y;
@@ -129,39 +152,10 @@ __device__ __forceinline__ float row_max(const float (&s)[N]) {
   return fmaxf(fmax3(m[0], m[1], m[2]), fmax3(fmax3(m[3], m[4], m[5]), m[6], m[7]));
 }
 
-// 2^x for a pair of values on the FMA and integer pipes, leaving the MUFU
-// unit to the other exponentials (the softmax is otherwise bound by MUFU
-// throughput, 16 ex2 per clock per SM).  Cody-Waite style reduction: adding
-// 1.5 * 2^23 rounds x to the nearest integer n (which also appears in the low
-// mantissa bits of the sum), f = x - n lies in [-1/2, 1/2], 2^f is a degree-3
-// polynomial fitted here to minimise the maximum relative error on that
-// interval (7.5e-5 with fp32 Horner evaluation), and n is added to the
-// exponent field.  Inputs are clamped to [-126, 64] (so the exponent field
-// cannot wrap); the results feed bf16 probabilities (relative precision
-// 3.9e-3).  Masked inputs (-inf) need exp2_scaled's masked path for an exact 0.
-__device__ __forceinline__ float2 exp2_poly2(float2 x) {
-  constexpr float kRound = 12582912.0f;  // 1.5 * 2^23
-  const float2 xc = make_float2(fminf(fmaxf(x.x, -126.0f), 64.0f), fminf(fmaxf(x.y, -126.0f), 64.0f));
-  const float2 t = __fadd2_rn(xc, make_float2(kRound, kRound));
-  const float2 n = __fadd2_rn(t, make_float2(-kRound, -kRound));
-  const float2 f = __fadd2_rn(xc, make_float2(-n.x, -n.y));
-  float2 q = __ffma2_rn(make_float2(5.517166853e-02f, 5.517166853e-02f), f,
-                        make_float2(2.426111251e-01f, 2.426111251e-01f));
-  q = __ffma2_rn(q, f, make_float2(6.932609677e-01f, 6.932609677e-01f));
-  q = __ffma2_rn(q, f, make_float2(9.999280572e-01f, 9.999280572e-01f));
-  // The rounded integer sits in the low mantissa bits of t: shift it into the
-  // exponent field (the constant part of t's bits cancels modulo 2^32).
-  constexpr int kBias = (int)(0x4B400000u << 23);
-  return make_float2(__int_as_float(__float_as_int(q.x) + (__float_as_int(t.x) << 23) - kBias),
-                     __int_as_float(__float_as_int(q.y) + (__float_as_int(t.y) << 23) - kBias));
-}
-
 // p = 2^(s * scale - shift) in place, two elements per packed FMA; returns
-// the sum of p.  kEmu of every 8 pairs use exp2_poly2, the rest MUFU ex2.
-// With `masked` (the row has masked keys in this tile) emulated results of
-// inputs below -126 are forced to exactly 0, as ex2 gives for -inf.
-template <int kEmu, int N>
-__device__ __forceinline__ float exp2_scaled(float (&s)[N], float scale, float shift, bool masked) {
+// the sum of p.
+template <int N>
+__device__ __forceinline__ float exp2_scaled(float (&s)[N], float scale, float shift) {
   const float2 sc = make_float2(scale, scale), sh = make_float2(-shift, -shift);
   float2 acc[4];
 #pragma unroll
@@ -169,17 +163,7 @@ __device__ __forceinline__ float exp2_scaled(float (&s)[N], float scale, float s
 #pragma unroll
   for (int c = 0; c < N; c += 2) {
     const float2 x = __ffma2_rn(make_float2(s[c], s[c + 1]), sc, sh);
-    float2 y;
-    if ((c / 2) % 8 < kEmu) {
-      y = exp2_poly2(x);
-      if (masked) {
-        y.x = x.x < -126.0f ? 0.0f : y.x;
-        y.y = x.y < -126.0f ? 0.0f : y.y;
-      }
-    } else {
-      y.x = ex2_approx(x.x);
-      y.y = ex2_approx(x.y);
-    }
+    const float2 y = make_float2(ex2_approx(x.x), ex2_approx(x.y));
     s[c] = y.x;
     s[c + 1] = y.y;
     acc[(c / 2) & 3] = __fadd2_rn(acc[(c / 2) & 3], y);
@@ -295,82 +279,33 @@ __device__ __forceinline__ void decode_unit(const AttnParams& p, int u, int& b, 
   h = bh % p.n_heads;
 }
 
-// One key tile of the CTA's stream, as the producer and the MMA warp need it.
-struct Tile {
-  int kb;     // key block
-  int z;      // batch * n_kv_heads + kv head (TMA outer coordinate of K and V)
-  int first;  // first tile of its unit
-};
-
-// The tiles of one CTA, unit after unit (units without any tile skipped).
-template <int BN, int MODE>
-struct TileStream {
-  int u, stride, z;
-  TileIter<BN, MODE> it;
-  int nkb, nfirst, have;
-  int bad;
-
-  __device__ __forceinline__ void open_next_unit(const AttnParams& p) {
-    for (;;) {
-      u += stride;
-      if (u >= p.n_units) {
-        have = 0;
-        return;
-      }
-      int b, h, qt;
-      decode_unit(p, u, b, h, qt);
-      const int kvh = h / p.group;
-      z = b * p.n_kv_heads + kvh;
-      it = make_iter<BN, MODE>(p, b, kvh, qt);
-      int bits;
-      if (it.next(nkb, bits)) {
-        nfirst = 1;
-        have = 1;
-        return;
-      }
-      bad |= it.bad;
-    }
-  }
-
-  __device__ __forceinline__ void start(const AttnParams& p) {
-    stride = gridDim.x;
-    u = blockIdx.x - stride;
-    bad = 0;
-    open_next_unit(p);
-  }
-
-  __device__ __forceinline__ bool next(const AttnParams& p, Tile& t) {
-    if (!have) return false;
-    t.kb = nkb;
-    t.z = z;
-    t.first = nfirst;
-    int bits;
-    if (it.next(nkb, bits)) {
-      nfirst = 0;
-    } else {
-      bad |= it.bad;
-      open_next_unit(p);
-    }
-    return true;
-  }
-};
-
 template <int RK, int RV>
-struct SharedBarriers {
+struct SharedState {
   uint64_t k_full[RK], k_empty[RK], v_full[RV], v_empty[RV];
-  // Barriers that a thread may reach late (after the producing side has
-  // already moved on by one item) exist once per buffer: a second completion
-  // of the same barrier then needs work that the waiting thread itself has
-  // not issued yet, so a parity wait can never skip a phase.
-  uint64_t q_full;       // Q tile landed in the staging buffer (TMA)
-  uint64_t q_tmem[2];    // Q copied into TMEM buffer b (8 softmax warps)
-  uint64_t s_full[2];    // S buffer b written (S thread commit)
-  uint64_t buf_free[2];  // P of buffer b consumed by its P V (P V thread commit)
-  uint64_t p_full[2];    // P of buffer b written into TMEM (8 softmax warps)
-  uint64_t o_full;       // a P V completed (P V thread commit)
-  uint64_t xch;          // the two softmax halves exchanged row values (8 warps)
+  uint64_t sched_full[kSchedSlots], sched_empty[kSchedSlots];
+  // A parity wait is exact only while the barrier is at most one phase away
+  // from the awaited one.  Barriers whose waiters may arrive late (after the
+  // next phase could complete) or early (before the previous phase has
+  // completed) therefore exist once per buffer: a second completion of the
+  // same barrier needs work that the waiter itself has not released yet, and
+  // its previous completion is implied by work the waiter has already seen.
+  uint64_t q_full;        // Q tile landed in the staging buffer (TMA)
+  uint64_t q_stage_free;  // staging buffer copied into TMEM (S thread commit)
+  uint64_t q_free[2];     // last S of a unit using Q buffer b completed (S thread commit)
+  uint64_t s_full[2];     // S buffer b written (S thread commit)
+  uint64_t buf_free[2];   // P of buffer b consumed by its P V (P V thread commit)
+  uint64_t p_full[2];     // P of buffer b written into TMEM (4 warps of warpgroup b)
+  uint64_t o_full[2];     // P V of a tile with P in buffer b completed (P V thread commit)
+  uint64_t o_free;        // both epilogue halves read O (8 softmax warps)
+  uint64_t m_pub[2][2];   // warpgroup w published its running max, slot = its tile count & 1
+  uint64_t l_pub[2];      // warpgroup w published its row-sum part of a unit
+  uint64_t l_ack[2];      // the other warpgroup read that part
+  uint64_t epi[2];        // the 4 warps of warpgroup w wrote their block-mass sums
   uint64_t s_done, pv_done;
-  float xbuf[2][2][128];  // [phase & 1][half][row]
+  int4 sched[kSchedSlots];
+  float mx[2][2][128];   // [warpgroup][slot][row] running max after a tile
+  float lx[2][128];      // [warpgroup][row] row-sum part at the end of a unit
+  float lm[2][128];      // [warpgroup][row] the max that part refers to
   uint32_t tmem_base;
   int abort;
 };
@@ -388,44 +323,88 @@ __device__ __forceinline__ void raise_status(const AttnParams& p, int* abort, in
 
 // ------------------------------------------------------------------ producer
 template <int D, int BN, int MODE>
-__device__ void attn_producer(const CUtensorMap* mapK, const CUtensorMap* mapV, const AttnParams& p, uint8_t* ring,
-                              SharedBarriers<AttnCfg<D, BN>::kRingK, AttnCfg<D, BN>::kRingV>& sb) {
+__device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, const CUtensorMap* mapV,
+                              const AttnParams& p, uint8_t* q_stage, uint8_t* ring,
+                              SharedState<AttnCfg<D, BN>::kRingK, AttnCfg<D, BN>::kRingV>& sb) {
   using C = AttnCfg<D, BN>;
   constexpr int RK = C::kRingK, RV = C::kRingV;
   uint8_t* k_ring = ring;
   uint8_t* v_ring = ring + RK * C::kKVBytes;
   volatile int* abort = &sb.abort;
-  TileStream<BN, MODE> st;
-  st.start(p);
-  int jk = 0, jv = 0;
+  int e = 0, jk = 0, jv = 0, nq = 0, bad = 0;
   bool ok = true;
-  auto load = [&](const CUtensorMap* map, uint8_t* base, uint64_t* full, uint64_t* empty, int R, int& j,
-                  const Tile& t) -> bool {
+  auto emit = [&](int kb, int u, int flags) -> bool {
+    const int slot = e % kSchedSlots;
+    if (e >= kSchedSlots && !mbar_wait(&sb.sched_empty[slot], ((e / kSchedSlots) - 1) & 1, abort)) return false;
+    sb.sched[slot] = make_int4(kb, u, flags, 0);
+    mbar_arrive(&sb.sched_full[slot]);  // release: the entry is visible to whoever acquires the phase
+    ++e;
+    return true;
+  };
+  auto load = [&](const CUtensorMap* map, uint8_t* base, uint64_t* full, uint64_t* empty, int R, int& j, int kb,
+                  int z) -> bool {
     const int slot = j % R;
     if (j >= R && !mbar_wait(&empty[slot], ((j / R) - 1) & 1, abort)) return false;
     mbar_arrive_expect_tx(&full[slot], C::kKVBytes);
     for (int i = 0; i < C::kBoxes; ++i)
-      tma_load_3d(base + slot * C::kKVBytes + i * BN * 128, map, &full[slot], 64 * i, t.kb * BN, t.z);
+      tma_load_3d(base + slot * C::kKVBytes + i * BN * 128, map, &full[slot], 64 * i, kb * BN, z);
     ++j;
     return true;
   };
-  Tile cur, nxt;
-  bool have = st.next(p, cur);
-  if (have && !load(mapK, k_ring, sb.k_full, sb.k_empty, RK, jk, cur)) ok = false;
-  while (have && ok) {
-    const bool more = st.next(p, nxt);
-    if (more && !load(mapK, k_ring, sb.k_full, sb.k_empty, RK, jk, nxt)) {
-      ok = false;
-      break;
+  const int G = gridDim.x, c = blockIdx.x;
+  int prev_kb = 0, prev_z = 0;
+  bool have_prev = false;
+  for (int k = 0; ok && k * G < p.n_units; ++k) {
+    const int u = k * G + ((k & 1) ? G - 1 - c : c);
+    if (u >= p.n_units) continue;  // only in the last, partial round
+    int b, h, qt;
+    decode_unit(p, u, b, h, qt);
+    const int kvh = h / p.group;
+    const int z = b * p.n_kv_heads + kvh;
+    auto it = make_iter<BN, MODE>(p, b, kvh, qt);
+    int kb, bits;
+    bool have = it.next(kb, bits);
+    if (!have && !emit(0, u, kEntEmpty)) ok = false;
+    bool first = true;
+    while (have && ok) {
+      int nkb, nbits;
+      const bool more = it.next(nkb, nbits);
+      if (!emit(kb, u, bits | (first ? kEntFirst : 0) | (more ? 0 : kEntLast))) {
+        ok = false;
+        break;
+      }
+      if (first) {
+        // The staging buffer is free once the previous unit's Q is in TMEM.
+        if (nq >= 1 && !mbar_wait(&sb.q_stage_free, (nq - 1) & 1, abort)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(&sb.q_full, C::kQBytes);
+        for (int i = 0; i < C::kBoxes; ++i)
+          tma_load_3d(q_stage + i * 128 * 128, mapQ, &sb.q_full, 64 * i, qt * 128, b * p.n_heads + h);
+        ++nq;
+      }
+      if (!load(mapK, k_ring, sb.k_full, sb.k_empty, RK, jk, kb, z)) {
+        ok = false;
+        break;
+      }
+      if (have_prev && !load(mapV, v_ring, sb.v_full, sb.v_empty, RV, jv, prev_kb, prev_z)) {
+        ok = false;
+        break;
+      }
+      prev_kb = kb;
+      prev_z = z;
+      have_prev = true;
+      kb = nkb;
+      bits = nbits;
+      have = more;
+      first = false;
     }
-    if (!load(mapV, v_ring, sb.v_full, sb.v_empty, RV, jv, cur)) {
-      ok = false;
-      break;
-    }
-    cur = nxt;
-    have = more;
+    bad |= it.bad;
   }
-  if (st.bad) atomicOr(p.status, kStatusBadSupport);
+  if (ok && have_prev && !load(mapV, v_ring, sb.v_full, sb.v_empty, RV, jv, prev_kb, prev_z)) ok = false;
+  if (ok && !emit(0, 0, kEntEnd)) ok = false;
+  if (bad) atomicOr(p.status, kStatusBadSupport);
   if (!ok) {
     raise_status(p, &sb.abort, kStatusTimeout);
     // Let every copy already issued land before the CTA's shared memory is
@@ -433,34 +412,70 @@ __device__ void attn_producer(const CUtensorMap* mapK, const CUtensorMap* mapV, 
     int never = 0;
     for (int t = max(0, jk - RK); t < jk; ++t) mbar_wait(&sb.k_full[t % RK], (t / RK) & 1, &never);
     for (int t = max(0, jv - RV); t < jv; ++t) mbar_wait(&sb.v_full[t % RV], (t / RV) & 1, &never);
+    if (nq > 0) mbar_wait(&sb.q_full, (nq - 1) & 1, &never);
   }
+}
+
+// Reads schedule entry e (single thread).
+template <class SS>
+__device__ __forceinline__ bool sched_read(SS& sb, int e, int4& ent, volatile int* abort) {
+  const int slot = e % kSchedSlots;
+  if (!mbar_wait(&sb.sched_full[slot], (e / kSchedSlots) & 1, abort)) return false;
+  ent = sb.sched[slot];
+  mbar_arrive(&sb.sched_empty[slot]);
+  return true;
 }
 
 // --------------------------------------------------------------- MMA issuers
 template <int D, int BN, int MODE>
-__device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* ring,
-                           SharedBarriers<AttnCfg<D, BN>::kRingK, AttnCfg<D, BN>::kRingV>& sb) {
+__device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* q_stage, uint8_t* ring,
+                           SharedState<AttnCfg<D, BN>::kRingK, AttnCfg<D, BN>::kRingV>& sb) {
   using C = AttnCfg<D, BN>;
   constexpr int RK = C::kRingK;
   volatile int* abort = &sb.abort;
   constexpr uint32_t idesc_s = idesc_bf16_f32(128, BN, false, false);
-  TileStream<BN, MODE> st;
-  st.start(p);
-  int n_q = 0;
+  int j = 0, nq = 0;
   uint32_t q_col = 0;  // TMEM column of the current unit's Q
   bool ok = true;
-  Tile t;
-  for (int j = 0; st.next(p, t); ++j) {
-    if (t.first) {
-      if (!mbar_wait(&sb.q_tmem[n_q & 1], (n_q >> 1) & 1, abort)) ok = false;
-      q_col = C::kTmemQ + (n_q & 1) * C::kTmemQCols;
-      ++n_q;
+  for (int e = 0;; ++e) {
+    int4 ent;
+    if (!sched_read(sb, e, ent, abort)) {
+      ok = false;
+      break;
+    }
+    if (ent.z & kEntEnd) break;
+    if (ent.z & kEntEmpty) continue;
+    if (ent.z & kEntFirst) {
+      // Q buffer nq & 1 was last read by the S products of unit nq - 2.
+      const int qb = nq & 1;
+      if (nq >= 2 && !mbar_wait(&sb.q_free[qb], ((nq >> 1) - 1) & 1, abort)) {
+        ok = false;
+        break;
+      }
+      if (!mbar_wait(&sb.q_full, nq & 1, abort)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after_sync();
+      q_col = C::kTmemQ + qb * C::kTmemQCols;
+      const uint32_t q_base = smem_u32(q_stage);
+#pragma unroll
+      for (int kk = 0; kk < D / 16; ++kk)
+        tmem_cp_128x256b(tmem + q_col + kk * 8,
+                         smem_desc_sw128(q_base + (kk >> 2) * (128 * 128) + (kk & 3) * 32, 16, 1024));
+      umma_commit(&sb.q_stage_free);
+      ++nq;
     }
     const int slot = j % RK;
-    if (ok && !mbar_wait(&sb.k_full[slot], (j / RK) & 1, abort)) ok = false;
+    if (!mbar_wait(&sb.k_full[slot], (j / RK) & 1, abort)) {
+      ok = false;
+      break;
+    }
     // S(j) overwrites the buffer that held P(j-2).
-    if (ok && j >= 2 && !mbar_wait(&sb.buf_free[j & 1], ((j >> 1) - 1) & 1, abort)) ok = false;
-    if (!ok) break;
+    if (j >= 2 && !mbar_wait(&sb.buf_free[j & 1], ((j >> 1) - 1) & 1, abort)) {
+      ok = false;
+      break;
+    }
     tc_fence_after_sync();
     const uint32_t s_col = C::kTmemS + (j & 1) * C::kTmemSCols;
     const uint64_t b0 = smem_desc_sw128(smem_u32(ring + slot * C::kKVBytes), 16, 1024);
@@ -473,9 +488,11 @@ __device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* ring,
     }
     umma_commit(&sb.s_full[j & 1]);
     umma_commit(&sb.k_empty[slot]);
+    if (ent.z & kEntLast) umma_commit(&sb.q_free[(nq - 1) & 1]);
+    ++j;
   }
   if (!ok) raise_status(p, &sb.abort, kStatusTimeout);
-  // Every MMA issued must have completed before TMEM is released.
+  // Every MMA and copy issued must have completed before TMEM is released.
   umma_commit(&sb.s_done);
   int never = 0;
   mbar_wait(&sb.s_done, 0, &never);
@@ -483,21 +500,41 @@ __device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* ring,
 
 template <int D, int BN, int MODE>
 __device__ void attn_mma_pv(const AttnParams& p, uint32_t tmem, uint8_t* ring,
-                            SharedBarriers<AttnCfg<D, BN>::kRingK, AttnCfg<D, BN>::kRingV>& sb) {
+                            SharedState<AttnCfg<D, BN>::kRingK, AttnCfg<D, BN>::kRingV>& sb) {
   using C = AttnCfg<D, BN>;
   constexpr int RK = C::kRingK, RV = C::kRingV;
   uint8_t* v_ring = ring + RK * C::kKVBytes;
   volatile int* abort = &sb.abort;
   constexpr uint32_t idesc_o = idesc_bf16_f32(128, D, false, true);
-  TileStream<BN, MODE> st;
-  st.start(p);
+  int j = 0, nu = 0;
   bool ok = true;
-  Tile t;
-  for (int j = 0; st.next(p, t); ++j) {
+  for (int e = 0;; ++e) {
+    int4 ent;
+    if (!sched_read(sb, e, ent, abort)) {
+      ok = false;
+      break;
+    }
+    if (ent.z & kEntEnd) break;
+    if (ent.z & kEntEmpty) continue;
+    const bool first = (ent.z & kEntFirst) != 0;
+    if (first) {
+      // The first P V of a unit overwrites O: both epilogue halves of the
+      // previous unit must have read it.
+      if (nu >= 1 && !mbar_wait(&sb.o_free, (nu - 1) & 1, abort)) {
+        ok = false;
+        break;
+      }
+      ++nu;
+    }
     const int slot = j % RV;
-    if (!mbar_wait(&sb.p_full[j & 1], (j >> 1) & 1, abort)) ok = false;
-    if (ok && !mbar_wait(&sb.v_full[slot], (j / RV) & 1, abort)) ok = false;
-    if (!ok) break;
+    if (!mbar_wait(&sb.p_full[j & 1], (j >> 1) & 1, abort)) {
+      ok = false;
+      break;
+    }
+    if (!mbar_wait(&sb.v_full[slot], (j / RV) & 1, abort)) {
+      ok = false;
+      break;
+    }
     tc_fence_after_sync();
     // P(j) sits in the first BN/2 columns of S buffer j & 1.
     const uint32_t p_col = C::kTmemS + (j & 1) * C::kTmemSCols;
@@ -505,10 +542,11 @@ __device__ void attn_mma_pv(const AttnParams& p, uint32_t tmem, uint8_t* ring,
 #pragma unroll 1
     for (int kk = 0; kk < BN / 16; ++kk)
       umma_bf16_ts(tmem + C::kTmemO, tmem + p_col + kk * 8, b0 + ((kk * 2048) >> 4), idesc_o,
-                   (t.first && kk == 0) ? 0u : 1u);
-    umma_commit(&sb.o_full);
+                   (first && kk == 0) ? 0u : 1u);
+    umma_commit(&sb.o_full[j & 1]);
     umma_commit(&sb.v_empty[slot]);
     umma_commit(&sb.buf_free[j & 1]);
+    ++j;
   }
   if (!ok) raise_status(p, &sb.abort, kStatusTimeout);
   umma_commit(&sb.pv_done);
@@ -516,335 +554,223 @@ __device__ void attn_mma_pv(const AttnParams& p, uint32_t tmem, uint8_t* ring,
   mbar_wait(&sb.pv_done, 0, &never);
 }
 
-// Issues the TMA load of the Q tile of unit u into the staging buffer.
-template <int D, int BN>
-__device__ __forceinline__ void load_q(const CUtensorMap* mapQ, const AttnParams& p, int u, uint8_t* q_stage,
-                                       uint64_t* bar) {
-  using C = AttnCfg<D, BN>;
-  int b, h, qt;
-  decode_unit(p, u, b, h, qt);
-  mbar_arrive_expect_tx(bar, C::kQBytes);
-  for (int i = 0; i < C::kBoxes; ++i)
-    tma_load_3d(q_stage + i * 128 * 128, mapQ, bar, 64 * i, qt * 128, b * p.n_heads + h);
-}
-
-// First unit at or after u (stepping by stride) that has at least one tile.
-template <int BN, int MODE>
-__device__ __forceinline__ int next_nonempty_unit(const AttnParams& p, int u, int stride) {
-  for (; u < p.n_units; u += stride) {
-    if (MODE != kSparse) return u;
-    int b, h, qt;
-    decode_unit(p, u, b, h, qt);
-    auto it = make_iter<BN, MODE>(p, b, h / p.group, qt);
-    int kb, bits;
-    if (it.next(kb, bits)) return u;
-  }
-  return INT_MAX;
-}
-
-// Loads this thread's kCols columns of an S tile (one or two 32-column
-// loads, one wait) and applies the causal / support masks.
+// Loads this thread's row of an S tile (kCols columns, one wait) and applies
+// the causal / support masks.
 template <int kCols>
-__device__ __forceinline__ void load_s_half(uint32_t addr, float (&s)[kCols], bool attend, int lim) {
+__device__ __forceinline__ void load_s_row(uint32_t addr, float (&s)[kCols], bool attend, int lim) {
+  static_assert(kCols == 64 || kCols == 128, "tile width");
   uint32_t va[32], vb[32];
   tmem_ld_32x32b_x32(addr, va);
-  if constexpr (kCols == 64) {
-    tmem_ld_32x32b_x32(addr + 32, vb);
-    tmem_ld_wait(va, vb);
+  tmem_ld_32x32b_x32(addr + 32, vb);
+  if constexpr (kCols == 128) {
+    uint32_t vc[32], vd[32];
+    tmem_ld_32x32b_x32(addr + 64, vc);
+    tmem_ld_32x32b_x32(addr + 96, vd);
+    tmem_ld_wait(va, vb);  // completes all four loads
+    reg_tie(vc);
+    reg_tie(vd);
+#pragma unroll
+    for (int e = 0; e < 32; ++e) {
+      s[64 + e] = __uint_as_float(vc[e]);
+      s[96 + e] = __uint_as_float(vd[e]);
+    }
   } else {
-    tmem_ld_wait(va);
+    tmem_ld_wait(va, vb);
   }
 #pragma unroll
-  for (int e = 0; e < 32; ++e) s[e] = __uint_as_float(va[e]);
-  if constexpr (kCols == 64) {
-#pragma unroll
-    for (int e = 0; e < 32; ++e) s[32 + e] = __uint_as_float(vb[e]);
+  for (int e = 0; e < 32; ++e) {
+    s[e] = __uint_as_float(va[e]);
+    s[32 + e] = __uint_as_float(vb[e]);
   }
-  if (!attend) {
+  // Keys with column c > lim are in the future of this row; a row that does
+  // not attend the tile masks every column.
+  const int lim_eff = attend ? lim : -1;
+  if (lim_eff < kCols - 1) {
 #pragma unroll
-    for (int c = 0; c < kCols; ++c) s[c] = -INFINITY;
-  } else if (lim < kCols - 1) {
-    // keys with column c > lim are in the future of this row
-#pragma unroll
-    for (int c = 0; c < kCols; ++c) s[c] = (c > lim) ? -INFINITY : s[c];
+    for (int c = 0; c < kCols; ++c) s[c] = (c > lim_eff) ? -INFINITY : s[c];
   }
 }
 
-// Exchange of one float per row between the two softmax halves: thread
-// (half, row) publishes v and gets its partner's value.  Double-buffered by
-// phase; bounded wait.
-template <class SB>
-__device__ __forceinline__ void half_publish(SB& sb, int phase, int half, int row, int lane, float v) {
-  sb.xbuf[phase & 1][half][row] = v;
-  __syncwarp();
-  if (lane == 0) mbar_arrive(&sb.xch);
-}
-
-template <class SB>
-__device__ __forceinline__ bool half_collect(SB& sb, int& phase, int half, int row, float& other,
-                                             volatile int* abort) {
-  if (!warp_wait(&sb.xch, phase & 1, abort)) return false;
-  other = sb.xbuf[phase & 1][half ^ 1][row];
-  ++phase;
-  return true;
-}
-
-template <class SB>
-__device__ __forceinline__ bool half_exchange(SB& sb, int& phase, int half, int row, int lane,
-                                              float v, float& other, volatile int* abort) {
-  half_publish(sb, phase, half, row, lane, v);
-  return half_collect(sb, phase, half, row, other, abort);
-}
+// What an epilogue half needs about its unit.
+struct EpiInfo {
+  int u;      // unit
+  int j0;     // tile counter of its first tile
+  int j1;     // tile counter of its last tile
+  int nu;     // index among this CTA's units with tiles
+  int n_kt;   // key tiles 0..n_kt-1 (dense variants)
+  float l, m; // this warpgroup's row-sum part and the max it refers to
+};
 
 // ------------------------------------------------------------------- softmax
-// Warpgroup `half` of the softmax owns, for every query row of the tile,
-// key columns [half*BN/2, (half+1)*BN/2) of S and output columns
-// [half*D/2, (half+1)*D/2) of O.
 template <int D, int BN, int MODE>
-__device__ void attn_softmax(const CUtensorMap* mapQ, const AttnParams& p, int half, uint32_t tmem,
-                             uint8_t* q_stage, SharedBarriers<AttnCfg<D, BN>::kRingK, AttnCfg<D, BN>::kRingV>& sb) {
+__device__ void attn_softmax(const AttnParams& p, int w, uint32_t tmem,
+                             SharedState<AttnCfg<D, BN>::kRingK, AttnCfg<D, BN>::kRingV>& sb) {
   using C = AttnCfg<D, BN>;
-  constexpr int kCols = BN / 2;  // S columns per half
-  constexpr int kOCols = D / 2;  // O columns per half
-  // Pairs of every 8 whose exponential runs on the FMA pipe; the block-mass
-  // variant keeps the hardware ex2 throughout for its sums.
-  constexpr int kEmu = (MODE == kDenseMass) ? 0 : WISE_EMU_PAIRS;
+  constexpr int kOHalf = D / 2;               // O columns per epilogue half
+  constexpr float kRescaleThreshold = 8.0f;   // log2 units: P stays <= 256
   volatile int* abort = &sb.abort;
-  const int r = threadIdx.x & 127;  // query row within the tile
+  const int r = threadIdx.x & 127;  // query row within the tile (TMEM lane)
   const int wq = r >> 5, lane = r & 31;
-  const bool leader = (half == 0 && r == 0);
   const uint32_t lane_tmem = tmem + ((uint32_t)(wq * 32) << 16);
-  constexpr float kRescaleThreshold = 8.0f;  // log2 units: P stays <= 256
-  const int G = gridDim.x;
-  // Per-CTA scratch: [n_blocks][2][128] log2 partial masses, then
-  // [2][4][n_blocks] per-warp column sums.
-  float* scratch = p.scratch + (size_t)blockIdx.x * p.n_blocks * 264;
-  float* warp_sums = scratch + (size_t)p.n_blocks * 256;
+  const uint32_t s_col = C::kTmemS + w * C::kTmemSCols;  // this warpgroup's S / P buffer
+  const int half_bit = (BN == 64) ? (1 << (r >> 6)) : 1;
+  // Per-CTA scratch (kDenseMass): this warpgroup's log2 partial masses
+  // [2 units][n_blocks / 2 + 1 tiles][128 rows] (tile t of a unit sits at
+  // t / 2), then [2 warpgroups][2][4 warps][n_blocks] per-warp column sums.
+  const int lc_tiles = p.n_blocks / 2 + 1;
+  float* cta_scratch = p.scratch + (size_t)blockIdx.x * scratch_floats_per_cta(p.n_blocks);
+  float* lc_own = cta_scratch + (size_t)w * 2 * lc_tiles * 128;
+  float* warp_sums = cta_scratch + (size_t)4 * lc_tiles * 128;
 
-  // Q pipeline: the staging buffer holds the Q of unit q_next; copy_next()
-  // moves it into TMEM buffer n_q & 1 and prefetches the following one.
-  int q_next = next_nonempty_unit<BN, MODE>(p, blockIdx.x, G);
-  int n_q = 0, x_phase = 0, j = 0;
-  if (leader && q_next != INT_MAX) load_q<D, BN>(mapQ, p, q_next, q_stage, &sb.q_full);
+  int j = 0, nu = 0, n_epi = 0;
+  int cur_u = 0, cur_j0 = 0, cur_row = 0;
+  float l_w = 0.0f, m_w = -INFINITY;  // this warpgroup's part of the row sum, relative to m_w
+  bool pend = false;
+  EpiInfo pe{};
   bool ok = true;
-  auto copy_next = [&]() -> bool {
-    if (!warp_wait(&sb.q_full, n_q & 1, abort)) return false;
-    const uint32_t q_col = C::kTmemQ + (n_q & 1) * C::kTmemQCols;
-    if (half < C::kBoxes) {
-      const uint32_t box = smem_u32(q_stage + half * 128 * 128) + r * 128;
-      uint32_t w[32];
+
+  // ---- one tile (j & 1 == w)
+  auto tile = [&](int kb, int bits, bool first) -> bool {
+    if (!warp_wait(&sb.s_full[w], (j >> 1) & 1, abort)) return false;
+    tc_fence_after_sync();
+    const bool attend = (bits & half_bit) != 0;
+    const int lim = cur_row - kb * BN;  // keys kb*BN + c with c > lim are in the future
+    float s[BN];
+    load_s_row<BN>(lane_tmem + s_col, s, attend, lim);
+    const float m_tile = row_max(s) * p.scale_log2;
+    // Running max after the previous tile (the other warpgroup's).
+    float m_prev = -INFINITY;
+    if (!first) {
+      const int jp = j - 1;
+      if (!warp_wait(&sb.m_pub[w ^ 1][(jp >> 1) & 1], (jp >> 2) & 1, abort)) return false;
+      m_prev = sb.mx[w ^ 1][(jp >> 1) & 1][r];
+    }
+    const float m_new = (m_tile > m_prev + kRescaleThreshold) ? m_tile : m_prev;
+    sb.mx[w][(j >> 1) & 1][r] = m_new;
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&sb.m_pub[w][(j >> 1) & 1]);
+    const float rowsum = exp2_scaled(s, p.scale_log2, m_new == -INFINITY ? 0.0f : m_new);
+    // P as bf16 pairs into the first BN/2 columns of this tile's S buffer;
+    // the stores complete while the bookkeeping below runs.
 #pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        const uint4 v = ld_shared_v4(box + ((c ^ (r & 7)) << 4));
-        w[4 * c + 0] = v.x;
-        w[4 * c + 1] = v.y;
-        w[4 * c + 2] = v.z;
-        w[4 * c + 3] = v.w;
+    for (int c = 0; c < BN / 32; ++c) {
+      uint32_t pw[16];
+#pragma unroll
+      for (int e = 0; e < 16; ++e) pw[e] = pack_bf16x2(s[32 * c + 2 * e], s[32 * c + 2 * e + 1]);
+      tmem_st_32x32b_x16(lane_tmem + s_col + 16 * c, pw);
+    }
+    if (m_new != m_w) {
+      l_w *= ex2_approx(m_w - m_new);  // 0 while m_w is -inf
+      m_w = m_new;
+    }
+    l_w += rowsum;
+    if (MODE == kDenseMass)
+      lc_own[((size_t)(nu & 1) * lc_tiles + ((j - cur_j0) >> 1)) * 128 + r] =
+          rowsum > 0.0f ? m_new + lg2_approx(rowsum) : -INFINITY;
+    // O (after P V(j-1)) is rescaled only when the max moved.  tcgen05.ld/st
+    // are warp-collective: the warp rescales together, lanes whose max did
+    // not move use a factor of 1.
+    const bool rescale = !first && m_new != m_prev && m_prev != -INFINITY;
+    if (__any_sync(0xffffffffu, rescale)) {
+      // P V(j-2) completed before S(j) could be issued, so o_full[(j-1) & 1]
+      // is at most one phase short of P V(j-1).
+      if (!warp_wait(&sb.o_full[(j - 1) & 1], ((j - 1) >> 1) & 1, abort)) return false;
+      tc_fence_after_sync();
+      const float f = rescale ? ex2_approx(m_prev - m_new) : 1.0f;
+#pragma unroll
+      for (int c = 0; c < D / 16; ++c) {
+        uint32_t v[16];
+        tmem_ld_32x32b_x16(lane_tmem + C::kTmemO + 16 * c, v);
+        tmem_ld_wait(v);
+#pragma unroll
+        for (int e = 0; e < 16; ++e) v[e] = __float_as_uint(__uint_as_float(v[e]) * f);
+        tmem_st_32x32b_x16(lane_tmem + C::kTmemO + 16 * c, v);
       }
-      tmem_st_32x32b_x32(lane_tmem + q_col + half * 32, w);
-      tmem_st_wait();
+    }
+    tmem_st_wait();
+    tc_fence_before_sync();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&sb.p_full[w]);
+    return true;
+  };
+
+  // ---- this warpgroup's half of a unit's epilogue
+  auto epilogue = [&](const EpiInfo& ei) -> bool {
+    const int x = w ^ 1;
+    if (!warp_wait(&sb.l_pub[x], ei.nu & 1, abort)) return false;
+    const float l_o = sb.lx[x][r], m_o = sb.lm[x][r];
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&sb.l_ack[x]);
+    // L handled the last tile: its max is the one O refers to, and E's max
+    // is at most that.
+    const bool is_L = ((ei.j1 & 1) == w);
+    const float lL = is_L ? ei.l : l_o, mL = is_L ? ei.m : m_o;
+    const float lE = is_L ? l_o : ei.l, mE = is_L ? m_o : ei.m;
+    const float l_row = (mE == -INFINITY) ? lL : lL + lE * ex2_approx(mE - mL);
+    // P V(j1-2) completed before S(j1), which the other part published
+    // above presupposes (or this warpgroup's tile j1 itself).
+    if (!warp_wait(&sb.o_full[ei.j1 & 1], (ei.j1 >> 1) & 1, abort)) return false;
+    tc_fence_after_sync();
+    int b, h, qt;
+    decode_unit(p, ei.u, b, h, qt);
+    const int row = qt * 128 + r;
+    const float inv_l = l_row > 0.0f ? 1.0f / l_row : 0.0f;
+    __nv_bfloat16* orow = p.O + ((size_t)(b * p.n_heads + h) * p.seqlen + row) * D + w * kOHalf;
+#pragma unroll
+    for (int c = 0; c < kOHalf / 16; ++c) {
+      uint32_t v[16];
+      tmem_ld_32x32b_x16(lane_tmem + C::kTmemO + w * kOHalf + 16 * c, v);
+      tmem_ld_wait(v);
+      uint32_t o[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e)
+        o[e] = pack_bf16x2(__uint_as_float(v[2 * e]) * inv_l, __uint_as_float(v[2 * e + 1]) * inv_l);
+      if (row < p.seqlen) {
+        uint4* dst = reinterpret_cast<uint4*>(orow + 16 * c);
+        dst[0] = make_uint4(o[0], o[1], o[2], o[3]);
+        dst[1] = make_uint4(o[4], o[5], o[6], o[7]);
+      }
     }
     tc_fence_before_sync();
     __syncwarp();
-    if (lane == 0) mbar_arrive(&sb.q_tmem[n_q & 1]);
-    const int following = next_nonempty_unit<BN, MODE>(p, q_next + G, G);
-    if (leader && following != INT_MAX) {
-      // Every warp has read the staging buffer once q_tmem completes.
-      if (!mbar_wait(&sb.q_tmem[n_q & 1], (n_q >> 1) & 1, abort)) return false;
-      load_q<D, BN>(mapQ, p, following, q_stage, &sb.q_full);
-    }
-    q_next = following;
-    ++n_q;
-    return true;
-  };
-  if (q_next != INT_MAX && !copy_next()) ok = false;
-
-  for (int u = blockIdx.x; u < p.n_units && ok; u += G) {
-    int b, h, qt;
-    decode_unit(p, u, b, h, qt);
-    auto it = make_iter<BN, MODE>(p, b, h / p.group, qt);
-    const int row = qt * 128 + r;
-    const int half_bit = (BN == 64) ? (1 << (r >> 6)) : 1;
-    float m_ref = -INFINITY, l = 0.0f;
-    int jj = 0, kb, bits, last_kb = -1;
-    bool have = it.next(kb, bits);
-    // The next unit's Q goes into the other TMEM buffer while this one runs.
-    if (have && q_next != INT_MAX && !copy_next()) {
-      ok = false;
-      break;
-    }
-    while (have) {
-      int nkb, nbits;
-      const bool more = it.next(nkb, nbits);
-      last_kb = kb;
-      const uint32_t s_col = C::kTmemS + (j & 1) * C::kTmemSCols;
-      if (!warp_wait(&sb.s_full[j & 1], (j >> 1) & 1, abort)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after_sync();
-      const int k0 = kb * BN + half * kCols;
-      const bool attend = (bits & half_bit) != 0;
-      const int lim = row - k0;  // keys k0 + c with c > lim are in the future
-      const uint32_t s_addr = lane_tmem + s_col + half * kCols;
-      float s[kCols];
-      load_s_half<kCols>(s_addr, s, attend, lim);
-      const float mx_local = row_max(s);
-      // The partner half's maximum is needed before the exponentials can be
-      // trusted; publish now and collect after them.  Past a unit's first
-      // tile the running max rarely moves, so the exponentials are computed
-      // speculatively against it and redone only where it did move.
-      half_publish(sb, x_phase, half, r, lane, mx_local);
-      const bool first_tile = (jj == 0);
-      const float m_old = m_ref;
-      float rowsum = 0.0f;
-      const bool masked = !attend || lim < kCols - 1;
-      if (!first_tile) rowsum = exp2_scaled<kEmu>(s, p.scale_log2, m_old == -INFINITY ? 0.0f : m_old, masked);
-      float mx_other;
-      if (!half_collect(sb, x_phase, half, r, mx_other, abort)) {
-        ok = false;
-        break;
-      }
-      const float m_tile = fmaxf(mx_local, mx_other) * p.scale_log2;
-      float alpha = 1.0f;
-      bool rescale = false;
-      if (m_tile > m_ref + kRescaleThreshold) {
-        alpha = ex2_approx(m_ref - m_tile);
-        rescale = (m_ref != -INFINITY);
-        m_ref = m_tile;
-        l *= alpha;
-      }
-      const float m_use = (m_ref == -INFINITY) ? 0.0f : m_ref;
-      if (first_tile) {
-        rowsum = exp2_scaled<kEmu>(s, p.scale_log2, m_use, masked);
-      } else if (__any_sync(0xffffffffu, m_ref != m_old)) {
-        // Redo the rows whose running max moved (S is still in TMEM).
-        float t[kCols];
-        load_s_half<kCols>(s_addr, t, attend, lim);
-        const float tsum = exp2_scaled<kEmu>(t, p.scale_log2, m_use, masked);
-        if (m_ref != m_old) {
-          rowsum = tsum;
-#pragma unroll
-          for (int c = 0; c < kCols; ++c) s[c] = t[c];
-        }
-      }
-      // P as bf16 pairs: keys [half*kCols, (half+1)*kCols) of the row go to
-      // columns [half*kCols/2, (half+1)*kCols/2) of this tile's S buffer.
-      // The stores complete while the bookkeeping below runs.
-#pragma unroll
-      for (int c = 0; c < kCols / 32; ++c) {
-        uint32_t w[16];
-#pragma unroll
-        for (int e = 0; e < 16; ++e) w[e] = pack_bf16x2(s[32 * c + 2 * e], s[32 * c + 2 * e + 1]);
-        tmem_st_32x32b_x16(lane_tmem + s_col + half * (kCols / 2) + 16 * c, w);
-      }
-      l += rowsum;  // this half's part of the row sum
-      if (MODE == kDenseMass)
-        scratch[((size_t)kb * 2 + half) * 128 + r] = rowsum > 0.0f ? m_ref + lg2_approx(rowsum) : -INFINITY;
-      // O is rescaled only after the previous P V completed.  tcgen05.ld/st
-      // are warp-collective: the warp rescales together, lanes whose max did
-      // not move use a factor of 1.
-      if (jj > 0 && __any_sync(0xffffffffu, rescale)) {
-        if (!warp_wait(&sb.o_full, (j - 1) & 1, abort)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after_sync();
-        const float f = rescale ? alpha : 1.0f;
-        const uint32_t o_col = C::kTmemO + half * kOCols;
-#pragma unroll
-        for (int c = 0; c < kOCols / 16; ++c) {
-          uint32_t v[16];
-          tmem_ld_32x32b_x16(lane_tmem + o_col + 16 * c, v);
-          tmem_ld_wait(v);
-#pragma unroll
-          for (int e = 0; e < 16; ++e) v[e] = __float_as_uint(__uint_as_float(v[e]) * f);
-          tmem_st_32x32b_x16(lane_tmem + o_col + 16 * c, v);
-        }
-      }
-      tmem_st_wait();
-      tc_fence_before_sync();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&sb.p_full[j & 1]);
-      ++j;
-      ++jj;
-      kb = nkb;
-      bits = nbits;
-      have = more;
-    }
-    if (!ok) break;
-    // ---- epilogue: O / l over both halves
-    float l_other = 0.0f;
-    if (!half_exchange(sb, x_phase, half, r, lane, l, l_other, abort)) {
-      ok = false;
-      break;
-    }
-    const float l_row = half == 0 ? l + l_other : l_other + l;  // same order in both halves
-    if (jj > 0) {
-      if (!warp_wait(&sb.o_full, (j - 1) & 1, abort)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after_sync();
-    }
-    const float inv_l = l_row > 0.0f ? 1.0f / l_row : 0.0f;
-    __nv_bfloat16* orow = p.O + ((size_t)(b * p.n_heads + h) * p.seqlen + row) * D + half * kOCols;
-#pragma unroll
-    for (int c = 0; c < kOCols / 16; ++c) {
-      uint32_t v[16];
-      if (jj > 0) {
-        tmem_ld_32x32b_x16(lane_tmem + C::kTmemO + half * kOCols + 16 * c, v);
-        tmem_ld_wait(v);
-      } else {
-#pragma unroll
-        for (int e = 0; e < 16; ++e) v[e] = 0u;
-      }
-      uint32_t w[8];
-#pragma unroll
-      for (int e = 0; e < 8; ++e)
-        w[e] = pack_bf16x2(__uint_as_float(v[2 * e]) * inv_l, __uint_as_float(v[2 * e + 1]) * inv_l);
-      if (row < p.seqlen) {
-        uint4* dst = reinterpret_cast<uint4*>(orow + 16 * c);
-        dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
-        dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
-      }
-    }
-    // ---- epilogue: block mass (Eq. 5)
-    if (MODE == kDenseMass) {
-      const float lse = m_ref + lg2_approx(l_row);
-      const int n_kt = last_kb + 1;
-      for (int t = 0; t < n_kt; ++t) {
-        const float lc = scratch[((size_t)t * 2 + half) * 128 + r];
+    if (lane == 0) mbar_arrive(&sb.o_free);
+    if constexpr (MODE == kDenseMass) {
+      // Block mass (Eq. 5) of this warpgroup's tiles: per row
+      // 2^(lc - lse), summed over the rows of each query block.
+      const float lse = mL + lg2_approx(l_row);
+      float* ws = warp_sums + (size_t)(w * 2 + (n_epi & 1)) * 4 * p.n_blocks;
+      const int n_kt = ei.n_kt;
+      // Dense variants: tile t of the unit is key block t.
+      for (int t = (w - ei.j0) & 1; t < n_kt; t += 2) {
+        const float lc = lc_own[((size_t)(ei.nu & 1) * lc_tiles + (t >> 1)) * 128 + r];
         float v = (row < p.seqlen) ? ex2_approx(lc - lse) : 0.0f;
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-        if (lane == 0) warp_sums[(half * 4 + wq) * p.n_blocks + t] = v;
+        if (lane == 0) ws[wq * p.n_blocks + t] = v;
       }
-      // The exchange barrier orders the eight warps' global writes before
-      // the reads below (release/acquire at CTA scope).
-      float unused;
-      if (!half_exchange(sb, x_phase, half, r, lane, 0.0f, unused, abort)) {
-        ok = false;
-        break;
-      }
+      // Orders the four warps' writes before the reads below (release /
+      // acquire at CTA scope).
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sb.epi[w]);
+      if (!warp_wait(&sb.epi[w], n_epi & 1, abort)) return false;
+      ++n_epi;
       constexpr int kHalves = 128 / BN;  // query blocks per tile
       const float inv_b = 1.0f / (float)BN;
-      const int tid = half * 128 + r;
-      for (int e = tid; e < kHalves * p.n_blocks; e += 256) {
+      for (int e = r; e < kHalves * p.n_blocks; e += 128) {
         const int hf = e / p.n_blocks, t = e % p.n_blocks;
         const int qblock = qt * kHalves + hf;
         if (qblock >= p.n_blocks) continue;
+        const bool own = (t < n_kt) ? (((ei.j0 + t) & 1) == w) : ((t & 1) == w);
+        if (!own) continue;
         float* out = p.blockmass + ((size_t)(b * p.n_heads + h) * p.n_blocks + qblock) * p.n_blocks + t;
         if (t < n_kt) {
           float sum = 0.0f;
           if (BN == 128) {
 #pragma unroll
-            for (int w = 0; w < 8; ++w) sum += warp_sums[w * p.n_blocks + t];
+            for (int q = 0; q < 4; ++q) sum += ws[q * p.n_blocks + t];
           } else {
 #pragma unroll
-            for (int hh = 0; hh < 2; ++hh)
-#pragma unroll
-              for (int w = 2 * hf; w < 2 * hf + 2; ++w) sum += warp_sums[(hh * 4 + w) * p.n_blocks + t];
+            for (int q = 2 * hf; q < 2 * hf + 2; ++q) sum += ws[q * p.n_blocks + t];
           }
           sum *= inv_b;
           *out = (p.step == 0) ? sum : *out + sum;
@@ -852,21 +778,84 @@ __device__ void attn_softmax(const CUtensorMap* mapQ, const AttnParams& p, int h
           *out = 0.0f;
         }
       }
-      // warp_sums is rewritten by the next unit.
-      if (!half_exchange(sb, x_phase, half, r, lane, 0.0f, unused, abort)) {
+    }
+    return true;
+  };
+
+  for (int e = 0; ok; ++e) {
+    const int slot = e % kSchedSlots;
+    if (!warp_wait(&sb.sched_full[slot], (e / kSchedSlots) & 1, abort)) {
+      ok = false;
+      break;
+    }
+    const int4 ent = sb.sched[slot];
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&sb.sched_empty[slot]);
+    const int fl = ent.z;
+    if (fl & kEntEnd) break;
+    if (fl & kEntEmpty) {
+      // No key tile: the rows of the unit attend nothing and are zero.
+      int b, h, qt;
+      decode_unit(p, ent.y, b, h, qt);
+      const int row = qt * 128 + r;
+      if (row < p.seqlen) {
+        uint4* dst = reinterpret_cast<uint4*>(p.O + ((size_t)(b * p.n_heads + h) * p.seqlen + row) * D + w * kOHalf);
+#pragma unroll
+        for (int c = 0; c < kOHalf / 8; ++c) dst[c] = make_uint4(0u, 0u, 0u, 0u);
+      }
+      continue;
+    }
+    if (fl & kEntFirst) {
+      int b, h, qt;
+      decode_unit(p, ent.y, b, h, qt);
+      cur_u = ent.y;
+      cur_j0 = j;
+      cur_row = qt * 128 + r;
+      l_w = 0.0f;
+      m_w = -INFINITY;
+    }
+    if ((j & 1) == w) {
+      if (!tile(ent.x, fl & 3, (fl & kEntFirst) != 0)) {
         ok = false;
         break;
       }
+      // A deferred epilogue half runs after this warpgroup's first tile of
+      // the following unit.
+      if (pend) {
+        if (!epilogue(pe)) {
+          ok = false;
+          break;
+        }
+        pend = false;
+      }
     }
-  }
-  if (!ok) {
-    raise_status(p, &sb.abort, kStatusTimeout);
-    if (leader && n_q > 0) {
-      // Let a Q copy still in flight land before shared memory is released.
-      int never = 0;
-      mbar_wait(&sb.q_full, n_q & 1, &never);
+    if (fl & kEntLast) {
+      // Publish this warpgroup's part of the row sum (once the other one has
+      // read the previous unit's part).
+      if (nu >= 1 && !warp_wait(&sb.l_ack[w], (nu - 1) & 1, abort)) {
+        ok = false;
+        break;
+      }
+      sb.lx[w][r] = l_w;
+      sb.lm[w][r] = m_w;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sb.l_pub[w]);
+      const EpiInfo ei{cur_u, cur_j0, j, nu, ent.x + 1, l_w, m_w};
+      ++nu;
+      if ((j & 1) == w) {
+        if (!epilogue(ei)) {
+          ok = false;
+          break;
+        }
+      } else {
+        pe = ei;
+        pend = true;
+      }
     }
+    ++j;
   }
+  if (ok && pend) ok = epilogue(pe);
+  if (!ok) raise_status(p, &sb.abort, kStatusTimeout);
 }
 
 // -------------------------------------------------------------------- kernel
@@ -875,11 +864,13 @@ __global__ void __launch_bounds__(AttnCfg<D, BN>::kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
                 const __grid_constant__ CUtensorMap mapV, const AttnParams p) {
   using C = AttnCfg<D, BN>;
+  using SS = SharedState<C::kRingK, C::kRingV>;
+  static_assert(sizeof(SS) <= C::kStaticReserve, "static shared memory");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* q_stage = smem;             // one Q tile
   uint8_t* ring = smem + C::kQBytes;   // kRing K/V entries
-  __shared__ SharedBarriers<C::kRingK, C::kRingV> sb;
+  __shared__ SS sb;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -892,15 +883,25 @@ __global__ void __launch_bounds__(AttnCfg<D, BN>::kThreads, 1)
       mbar_init(&sb.v_full[i], 1);
       mbar_init(&sb.v_empty[i], 1);
     }
+    for (int i = 0; i < kSchedSlots; ++i) {
+      mbar_init(&sb.sched_full[i], 1);
+      mbar_init(&sb.sched_empty[i], kSchedReaders);
+    }
     mbar_init(&sb.q_full, 1);
+    mbar_init(&sb.q_stage_free, 1);
     for (int b = 0; b < 2; ++b) {
-      mbar_init(&sb.q_tmem[b], 8);
+      mbar_init(&sb.q_free[b], 1);
       mbar_init(&sb.s_full[b], 1);
       mbar_init(&sb.buf_free[b], 1);
-      mbar_init(&sb.p_full[b], 8);
+      mbar_init(&sb.p_full[b], 4);
+      mbar_init(&sb.m_pub[b][0], 4);
+      mbar_init(&sb.m_pub[b][1], 4);
+      mbar_init(&sb.l_pub[b], 4);
+      mbar_init(&sb.l_ack[b], 4);
+      mbar_init(&sb.epi[b], 4);
+      mbar_init(&sb.o_full[b], 1);
     }
-    mbar_init(&sb.o_full, 1);
-    mbar_init(&sb.xch, 8);
+    mbar_init(&sb.o_free, 8);
     mbar_init(&sb.s_done, 1);
     mbar_init(&sb.pv_done, 1);
     fence_mbar_init();
@@ -920,13 +921,17 @@ __global__ void __launch_bounds__(AttnCfg<D, BN>::kThreads, 1)
   const uint32_t tmem = sb.tmem_base;
 
   if (warp < 8) {
-    attn_softmax<D, BN, MODE>(&mapQ, p, warp >> 2, tmem, q_stage, sb);
-  } else if (warp == C::kProducerWarp) {
-    if (lane == 0) attn_producer<D, BN, MODE>(&mapK, &mapV, p, ring, sb);
-  } else if (warp == C::kMmaSWarp) {
-    if (lane == 0) attn_mma_s<D, BN, MODE>(p, tmem, ring, sb);
-  } else if (warp == C::kMmaPVWarp) {
-    if (lane == 0) attn_mma_pv<D, BN, MODE>(p, tmem, ring, sb);
+    warpgroup_reg_inc<C::kRegsSoftmax>();
+    attn_softmax<D, BN, MODE>(p, warp >> 2, tmem, sb);
+  } else {
+    warpgroup_reg_dec<C::kRegsOther>();
+    if (warp == C::kProducerWarp) {
+      if (lane == 0) attn_producer<D, BN, MODE>(&mapQ, &mapK, &mapV, p, q_stage, ring, sb);
+    } else if (warp == C::kMmaSWarp) {
+      if (lane == 0) attn_mma_s<D, BN, MODE>(p, tmem, q_stage, ring, sb);
+    } else if (warp == C::kMmaPVWarp) {
+      if (lane == 0) attn_mma_pv<D, BN, MODE>(p, tmem, ring, sb);
+    }
   }
 
   __syncwarp();

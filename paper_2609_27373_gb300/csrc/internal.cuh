@@ -12,6 +12,15 @@ namespace wise {
 
 enum AttnMode : int { kDense = 0, kDenseMass = 1, kSparse = 2 };
 
+// Per-CTA scratch of kDenseMass, in floats, for n_blocks key blocks:
+// log2 partial masses [2 warpgroups][2 units][n_blocks / 2 + 1 tiles][128
+// rows] (a warpgroup handles every other tile of a unit, and keeps the
+// previous unit's values until its epilogue has read them), then per-warp
+// column sums [2 warpgroups][2][4 warps][n_blocks].
+__host__ __device__ constexpr size_t scratch_floats_per_cta(int n_blocks) {
+  return (size_t)512 * (n_blocks / 2 + 1) + (size_t)16 * n_blocks;
+}
+
 // Bits of the per-device status word.
 constexpr int kStatusTimeout = 1;
 constexpr int kStatusBadSupport = 2;
@@ -28,8 +37,7 @@ struct AttnParams {
   const int32_t* idx;     // kSparse
   const int32_t* counts;  // kSparse
   int cap;                // kSparse
-  float* scratch;         // kDenseMass: per CTA [n_blocks][2][128] log2 partial masses followed
-                          // by [2][4][n_blocks] per-warp sums
+  float* scratch;         // kDenseMass: scratch_floats_per_cta(n_blocks) floats per CTA
   int* status;
 };
 

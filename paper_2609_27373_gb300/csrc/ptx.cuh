@@ -223,6 +223,28 @@ __device__ __forceinline__ void tmem_ld_wait(uint32_t (&a)[32], uint32_t (&b)[32
       : "memory");
 }
 
+// Makes the 32 registers look redefined at this point, so that no use of
+// them is scheduled ahead of it (pairs with an earlier tcgen05.wait::ld that
+// covered their load).
+__device__ __forceinline__ void reg_tie(uint32_t (&r)[32]) {
+  asm volatile(""
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                 "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
+                 "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]),
+                 "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]),
+                 "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
+               :
+               : "memory");
+}
+
+// Copies a 128-row x 32-byte slice of a shared-memory operand (described by
+// a matrix descriptor, as for an MMA operand) into 8 TMEM columns: row i goes
+// to lane i.  Asynchronous; ordered before later tcgen05.mma of the same
+// thread, completion tracked by tcgen05.commit.
+__device__ __forceinline__ void tmem_cp_128x256b(uint32_t taddr, uint64_t desc) {
+  asm volatile("tcgen05.cp.cta_group::1.128x256b [%0], %1;" ::"r"(taddr), "l"(desc) : "memory");
+}
+
 __device__ __forceinline__ void tmem_st_32x32b_x32(uint32_t taddr, const uint32_t (&r)[32]) {
   asm volatile(
       "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "

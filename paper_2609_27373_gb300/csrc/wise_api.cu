@@ -178,7 +178,7 @@ int launch_attention(const wise_shape_t* sh, const void* Q, const void* K, const
   if (mode == kDenseMass) {
     // Per CTA: [nKB][2][128] log2 partial masses and [2][4][nKB] per-warp
     // sums.
-    const size_t need = (size_t)L.grid * n_blocks * 264 * sizeof(float);
+    const size_t need = (size_t)L.grid * scratch_floats_per_cta(n_blocks) * sizeof(float);
     if (caller_scratch) {
       if (need > caller_scratch_bytes) return WISE_ERR_UNSUPPORTED;
       p.scratch = caller_scratch;

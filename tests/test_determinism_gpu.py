@@ -43,7 +43,8 @@ def test_repeated_launches_are_bit_identical(B, H, Hkv, L, D, blk):
             # the sparse kernel with every block equals the dense kernel
             assert torch.equal(Od.view(torch.int16), Op.view(torch.int16))
         else:
-            for x, y in zip(outs, ref):
-                assert torch.equal(x.view(torch.int32 if x.dtype == torch.float32 else torch.int16),
-                                   y.view(torch.int32 if y.dtype == torch.float32 else torch.int16))
+            names = ["dense+mass O", "block mass", "dense O", "sparse O", "all-blocks sparse O"]
+            for name, x, y in zip(names, outs, ref):
+                iv = torch.int32 if x.dtype == torch.float32 else torch.int16
+                assert torch.equal(x.view(iv), y.view(iv)), f"rep {rep}: {name} differs from rep 0"
     assert wise.wise_get_status() == wise.WISE_OK

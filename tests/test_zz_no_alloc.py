@@ -44,7 +44,7 @@ def test_noalloc_matches_the_allocating_entry_point_on_two_calls(B, H, Hkv, L, D
 
 
 def test_noalloc_rejects_a_problem_beyond_its_scratch():
-    # 32 heads x 256 query tiles >= one CTA per SM, each needing 256 blocks * 512 B:
+    # 32 heads x 256 query tiles >= one CTA per SM, each needing about 256 blocks * 1 KB:
     # far more than the 8 MiB array.
     shape = wise.Shape(1, 32768, 32, 8, 128, 128)
     Q = torch.zeros((1, 32, 32768, 128), dtype=torch.bfloat16, device="cuda")
