@@ -23,9 +23,12 @@
 //                shared memory (K-major);
 //   O += P V     P written by the softmax into TMEM, V from shared memory
 //                (MN-major).
-// TMEM (512 columns): Q double-buffered across units (2 x 64 columns), S
-// double-buffered across tiles (2 x 128 columns, P overwrites the first BN/2
-// columns of its S), O (128 columns).
+// TMEM (512 columns): Q (64 columns), P (64 columns), S double-buffered
+// across tiles (2 x 128 columns), O (128 columns).  S(j+2) is issued as soon
+// as the softmax has read S(j) into registers, so the S product runs up to two
+// tiles ahead and never waits for a P V; P(j) waits for P V(j-1), which
+// normally completed while the softmax of tile j ran.  The Q of the next unit
+// is copied in once the last S product of the current unit has completed.
 //
 // Warp roles (384 threads; warp 11 only completes warpgroup 2):
 //   warp 8     producer.  Walks the CTA's units, validates the support lists,
@@ -35,13 +38,13 @@
 //              TMA loads of Q (staging buffer), K (ring of kRingK) and V (ring
 //              of kRingV) in the order Q, K(0), K(1), V(0), K(2), V(1), ...
 //   warp 9     S issuer: copies each unit's Q into TMEM and issues
-//              S(j) = Q K(j)^T into S buffer j & 1.
+//              S(j) = Q K(j)^T into S buffer j & 1 once S(j-2) has been read.
 //   warp 10    P V issuer: O += P(j) V(j) once the softmax has written P(j).
 //              A tcgen05.mma issue blocks its thread while the tensor core
 //              drains earlier instructions, so the two products are issued
 //              from two threads.
 //   warps 0-3 and 4-7  softmax warpgroups 0 and 1.  Warpgroup w handles the
-//              tiles j with j & 1 == w (so it always uses S buffer w); thread
+//              tiles j with j & 1 == w (so it always reads S buffer w); thread
 //              t of a warpgroup owns query row t (= TMEM lane t) and the whole
 //              row of each of its tiles.  The online softmax runs in the log2
 //              domain with one running max m per row shared by both
@@ -90,9 +93,9 @@ struct AttnCfg {
   // At least 116 KB so that a single CTA resides per SM (it owns all 512
   // TMEM columns).
   static constexpr int kSmemLaunch = kSmemBytes > 116 * 1024 ? kSmemBytes : 116 * 1024;
-  static constexpr uint32_t kTmemQ = 0;       // two Q buffers
-  static constexpr uint32_t kTmemQCols = 64;  // 128 bf16 of Q per row
-  static constexpr uint32_t kTmemS = 128;     // two S/P buffers
+  static constexpr uint32_t kTmemQ = 0;       // Q: 128 bf16 per row
+  static constexpr uint32_t kTmemP = 64;      // P: 128 bf16 per row
+  static constexpr uint32_t kTmemS = 128;     // two S buffers
   static constexpr uint32_t kTmemSCols = 128;
   static constexpr uint32_t kTmemO = 384;     // O accumulator
   static constexpr uint32_t kTmemCols = 512;
@@ -291,11 +294,11 @@ struct SharedState {
   // its previous completion is implied by work the waiter has already seen.
   uint64_t q_full;        // Q tile landed in the staging buffer (TMA)
   uint64_t q_stage_free;  // staging buffer copied into TMEM (S thread commit)
-  uint64_t q_free[2];     // last S of a unit using Q buffer b completed (S thread commit)
+  uint64_t q_free;        // last S of a unit completed (S thread commit)
   uint64_t s_full[2];     // S buffer b written (S thread commit)
-  uint64_t buf_free[2];   // P of buffer b consumed by its P V (P V thread commit)
-  uint64_t p_full[2];     // P of buffer b written into TMEM (4 warps of warpgroup b)
-  uint64_t o_full[2];     // P V of a tile with P in buffer b completed (P V thread commit)
+  uint64_t s_free[2];     // S buffer b read by its softmax warpgroup (4 warps)
+  uint64_t p_full[2];     // P(j) written, j & 1 == b (4 warps of warpgroup b)
+  uint64_t o_full[2];     // P V(j) completed, j & 1 == b (P V thread commit); also frees P
   uint64_t o_free;        // both epilogue halves read O (8 softmax warps)
   uint64_t m_pub[2][2];   // warpgroup w published its running max, slot = its tile count & 1
   uint64_t l_pub[2];      // warpgroup w published its row-sum part of a unit
@@ -435,7 +438,6 @@ __device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* q_stage,
   volatile int* abort = &sb.abort;
   constexpr uint32_t idesc_s = idesc_bf16_f32(128, BN, false, false);
   int j = 0, nq = 0;
-  uint32_t q_col = 0;  // TMEM column of the current unit's Q
   bool ok = true;
   for (int e = 0;; ++e) {
     int4 ent;
@@ -446,9 +448,8 @@ __device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* q_stage,
     if (ent.z & kEntEnd) break;
     if (ent.z & kEntEmpty) continue;
     if (ent.z & kEntFirst) {
-      // Q buffer nq & 1 was last read by the S products of unit nq - 2.
-      const int qb = nq & 1;
-      if (nq >= 2 && !mbar_wait(&sb.q_free[qb], ((nq >> 1) - 1) & 1, abort)) {
+      // Q in TMEM was last read by the S products of unit nq - 1.
+      if (nq >= 1 && !mbar_wait(&sb.q_free, (nq - 1) & 1, abort)) {
         ok = false;
         break;
       }
@@ -457,11 +458,10 @@ __device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* q_stage,
         break;
       }
       tc_fence_after_sync();
-      q_col = C::kTmemQ + qb * C::kTmemQCols;
       const uint32_t q_base = smem_u32(q_stage);
 #pragma unroll
       for (int kk = 0; kk < D / 16; ++kk)
-        tmem_cp_128x256b(tmem + q_col + kk * 8,
+        tmem_cp_128x256b(tmem + C::kTmemQ + kk * 8,
                          smem_desc_sw128(q_base + (kk >> 2) * (128 * 128) + (kk & 3) * 32, 16, 1024));
       umma_commit(&sb.q_stage_free);
       ++nq;
@@ -471,8 +471,8 @@ __device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* q_stage,
       ok = false;
       break;
     }
-    // S(j) overwrites the buffer that held P(j-2).
-    if (j >= 2 && !mbar_wait(&sb.buf_free[j & 1], ((j >> 1) - 1) & 1, abort)) {
+    // S(j) overwrites S(j-2): its softmax warpgroup must have read it.
+    if (j >= 2 && !mbar_wait(&sb.s_free[j & 1], ((j >> 1) - 1) & 1, abort)) {
       ok = false;
       break;
     }
@@ -484,11 +484,11 @@ __device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* q_stage,
       // K step kk: 8 TMEM columns of Q; shared-memory descriptors of later
       // steps differ only in the start address field (address >> 4).
       const uint32_t b_off = ((kk >> 2) * (BN * 128) + (kk & 3) * 32) >> 4;
-      umma_bf16_ts(tmem + s_col, tmem + q_col + kk * 8, b0 + b_off, idesc_s, kk > 0 ? 1u : 0u);
+      umma_bf16_ts(tmem + s_col, tmem + C::kTmemQ + kk * 8, b0 + b_off, idesc_s, kk > 0 ? 1u : 0u);
     }
     umma_commit(&sb.s_full[j & 1]);
     umma_commit(&sb.k_empty[slot]);
-    if (ent.z & kEntLast) umma_commit(&sb.q_free[(nq - 1) & 1]);
+    if (ent.z & kEntLast) umma_commit(&sb.q_free);
     ++j;
   }
   if (!ok) raise_status(p, &sb.abort, kStatusTimeout);
@@ -536,8 +536,7 @@ __device__ void attn_mma_pv(const AttnParams& p, uint32_t tmem, uint8_t* ring,
       break;
     }
     tc_fence_after_sync();
-    // P(j) sits in the first BN/2 columns of S buffer j & 1.
-    const uint32_t p_col = C::kTmemS + (j & 1) * C::kTmemSCols;
+    const uint32_t p_col = C::kTmemP;
     const uint64_t b0 = smem_desc_sw128(smem_u32(v_ring + slot * C::kKVBytes), BN * 128, 1024);
 #pragma unroll 1
     for (int kk = 0; kk < BN / 16; ++kk)
@@ -545,7 +544,6 @@ __device__ void attn_mma_pv(const AttnParams& p, uint32_t tmem, uint8_t* ring,
                    (first && kk == 0) ? 0u : 1u);
     umma_commit(&sb.o_full[j & 1]);
     umma_commit(&sb.v_empty[slot]);
-    umma_commit(&sb.buf_free[j & 1]);
     ++j;
   }
   if (!ok) raise_status(p, &sb.abort, kStatusTimeout);
@@ -612,7 +610,8 @@ __device__ void attn_softmax(const AttnParams& p, int w, uint32_t tmem,
   const int r = threadIdx.x & 127;  // query row within the tile (TMEM lane)
   const int wq = r >> 5, lane = r & 31;
   const uint32_t lane_tmem = tmem + ((uint32_t)(wq * 32) << 16);
-  const uint32_t s_col = C::kTmemS + w * C::kTmemSCols;  // this warpgroup's S / P buffer
+  const uint32_t s_col = C::kTmemS + w * C::kTmemSCols;  // this warpgroup's S buffer
+  const uint32_t p_col = C::kTmemP;
   const int half_bit = (BN == 64) ? (1 << (r >> 6)) : 1;
   // Per-CTA scratch (kDenseMass): this warpgroup's log2 partial masses
   // [2 units][n_blocks / 2 + 1 tiles][128 rows] (tile t of a unit sits at
@@ -637,6 +636,10 @@ __device__ void attn_softmax(const AttnParams& p, int w, uint32_t tmem,
     const int lim = cur_row - kb * BN;  // keys kb*BN + c with c > lim are in the future
     float s[BN];
     load_s_row<BN>(lane_tmem + s_col, s, attend, lim);
+    // S(j) is in registers: S(j+2) may overwrite it.
+    tc_fence_before_sync();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&sb.s_free[w]);
     const float m_tile = row_max(s) * p.scale_log2;
     // Running max after the previous tile (the other warpgroup's).
     float m_prev = -INFINITY;
@@ -650,14 +653,19 @@ __device__ void attn_softmax(const AttnParams& p, int w, uint32_t tmem,
     __syncwarp();
     if (lane == 0) mbar_arrive(&sb.m_pub[w][(j >> 1) & 1]);
     const float rowsum = exp2_scaled(s, p.scale_log2, m_new == -INFINITY ? 0.0f : m_new);
-    // P as bf16 pairs into the first BN/2 columns of this tile's S buffer;
-    // the stores complete while the bookkeeping below runs.
+    // P was last read by P V(j-1), and O must have received it before a
+    // rescale.  P V(j-2) completed before tile j-1's P was written, which this
+    // warpgroup's own previous wait (or the exchange of the running max)
+    // implies, so o_full[(j-1) & 1] is at most one phase short of P V(j-1).
+    if (j >= 1 && !warp_wait(&sb.o_full[(j - 1) & 1], ((j - 1) >> 1) & 1, abort)) return false;
+    tc_fence_after_sync();
+    // P as bf16 pairs; the stores complete while the bookkeeping below runs.
 #pragma unroll
     for (int c = 0; c < BN / 32; ++c) {
       uint32_t pw[16];
 #pragma unroll
       for (int e = 0; e < 16; ++e) pw[e] = pack_bf16x2(s[32 * c + 2 * e], s[32 * c + 2 * e + 1]);
-      tmem_st_32x32b_x16(lane_tmem + s_col + 16 * c, pw);
+      tmem_st_32x32b_x16(lane_tmem + p_col + 16 * c, pw);
     }
     if (m_new != m_w) {
       l_w *= ex2_approx(m_w - m_new);  // 0 while m_w is -inf
@@ -672,10 +680,6 @@ __device__ void attn_softmax(const AttnParams& p, int w, uint32_t tmem,
     // not move use a factor of 1.
     const bool rescale = !first && m_new != m_prev && m_prev != -INFINITY;
     if (__any_sync(0xffffffffu, rescale)) {
-      // P V(j-2) completed before S(j) could be issued, so o_full[(j-1) & 1]
-      // is at most one phase short of P V(j-1).
-      if (!warp_wait(&sb.o_full[(j - 1) & 1], ((j - 1) >> 1) & 1, abort)) return false;
-      tc_fence_after_sync();
       const float f = rescale ? ex2_approx(m_prev - m_new) : 1.0f;
 #pragma unroll
       for (int c = 0; c < D / 16; ++c) {
@@ -707,8 +711,8 @@ __device__ void attn_softmax(const AttnParams& p, int w, uint32_t tmem,
     const float lL = is_L ? ei.l : l_o, mL = is_L ? ei.m : m_o;
     const float lE = is_L ? l_o : ei.l, mE = is_L ? m_o : ei.m;
     const float l_row = (mE == -INFINITY) ? lL : lL + lE * ex2_approx(mE - mL);
-    // P V(j1-2) completed before S(j1), which the other part published
-    // above presupposes (or this warpgroup's tile j1 itself).
+    // P V(j1-2) completed before P(j1) was written, which the other part
+    // published above presupposes (or this warpgroup's tile j1 itself).
     if (!warp_wait(&sb.o_full[ei.j1 & 1], (ei.j1 >> 1) & 1, abort)) return false;
     tc_fence_after_sync();
     int b, h, qt;
@@ -889,10 +893,10 @@ __global__ void __launch_bounds__(AttnCfg<D, BN>::kThreads, 1)
     }
     mbar_init(&sb.q_full, 1);
     mbar_init(&sb.q_stage_free, 1);
+    mbar_init(&sb.q_free, 1);
     for (int b = 0; b < 2; ++b) {
-      mbar_init(&sb.q_free[b], 1);
       mbar_init(&sb.s_full[b], 1);
-      mbar_init(&sb.buf_free[b], 1);
+      mbar_init(&sb.s_free[b], 4);
       mbar_init(&sb.p_full[b], 4);
       mbar_init(&sb.m_pub[b][0], 4);
       mbar_init(&sb.m_pub[b][1], 4);
