@@ -32,9 +32,11 @@
 //
 // Warp roles (384 threads; warp 11 only completes warpgroup 2):
 //   warp 8     producer.  Walks the CTA's units, validates the support lists,
-//              and publishes the tile schedule (one entry per tile, plus
-//              markers for units without tiles and for the end) in a
-//              shared-memory ring that every other role reads; issues the
+//              and publishes the tile schedule in three shared-memory rings:
+//              ring w (w = 0, 1) holds the tiles j with j & 1 == w for softmax
+//              warpgroup w (ring 0 also the units without tiles), ring 2 every
+//              tile for the two MMA threads, and each ring ends with an end
+//              marker; issues the
 //              TMA loads of Q (staging buffer), K (ring of kRingK) and V (ring
 //              of kRingV) in the order Q, K(0), K(1), V(0), K(2), V(1), ...
 //   warp 9     S issuer: copies each unit's Q into TMEM and issues
@@ -55,13 +57,12 @@
 //              sum; the two parts are combined at the end of the unit.  Since
 //              the two warpgroups work on different tiles, one computes
 //              exponentials while the other loads S or writes P.
-//   Epilogue.  O / l goes to global memory in two column halves, one per
-//              warpgroup.  The warpgroup that handled the unit's last tile
-//              writes its half at once; the other one first runs its tile of
-//              the next unit (its next tile always is that unit's first) and
-//              then writes its half, so that the tensor core receives the
-//              next P while the epilogue runs.  The first P V of a unit waits
-//              until both halves have read O.
+//   Epilogue.  The warpgroup that handled the unit's last tile (L) writes
+//              O / l to global memory (and, for kDenseMass, the block
+//              masses); the other one (E) only publishes its part of the row
+//              sum and goes on with the next unit's first tile, which is
+//              always its own.  The first P V of a unit waits until L has
+//              read O.
 //
 // Every wait is bounded (kWaitLimitNs); a wait that runs out sets the status
 // word and an abort flag, and every role unwinds.
@@ -82,14 +83,17 @@ struct AttnCfg {
   static constexpr int kQBytes = kBoxes * 128 * 128;    // one 128-row Q tile (staging)
   static constexpr int kKVBytes = kBoxes * BN * 128;    // one BN-row K or V tile (one ring entry)
   // Static shared memory (barriers, schedule ring, row exchange buffers).
-  static constexpr int kStaticReserve = 6 * 1024;
+  static constexpr int kStaticReserve = 7 * 1024;
   // Dynamic shared memory available after the 1024-byte alignment slack.
   static constexpr int kBudget = 227 * 1024 - 1024 - kStaticReserve;
-  static constexpr int kRingFit = (kBudget - kQBytes) / kKVBytes;
+  // Epilogue staging: per softmax warp of L, 32 rows x 64 columns of O
+  // (one 128-byte-swizzled TMA box).
+  static constexpr int kOutBytes = 4 * 32 * 128;
+  static constexpr int kRingFit = (kBudget - kQBytes - kOutBytes) / kKVBytes;
   static constexpr int kRing = kRingFit > 12 ? 12 : kRingFit;
   static constexpr int kRingK = (kRing + 1) / 2;  // K tiles (consumed by S)
   static constexpr int kRingV = kRing / 2;        // V tiles (consumed by P V)
-  static constexpr int kSmemBytes = kQBytes + kRing * kKVBytes + 1024;
+  static constexpr int kSmemBytes = kQBytes + kRing * kKVBytes + kOutBytes + 1024;
   // At least 116 KB so that a single CTA resides per SM (it owns all 512
   // TMEM columns).
   static constexpr int kSmemLaunch = kSmemBytes > 116 * 1024 ? kSmemBytes : 116 * 1024;
@@ -113,15 +117,18 @@ struct AttnCfg {
   static_assert(256 * kRegsSoftmax + 128 * kRegsOther <= kThreads * 168, "register split");
 };
 
-// Tile schedule ring.  Entry = {key block, unit, flags, 0}; the low two flag
-// bits say which 64-row halves of the query tile attend the key block.
-constexpr int kSchedSlots = 32;
-constexpr int kEntFirst = 4;   // first tile of its unit
-constexpr int kEntLast = 8;    // last tile of its unit
-constexpr int kEntEmpty = 16;  // unit without tiles (its output rows are zero)
-constexpr int kEntEnd = 32;    // no more units for this CTA
-// Readers of every entry: the two MMA threads and the eight softmax warps.
-constexpr int kSchedReaders = 10;
+// Tile schedule rings.  Entry = {key block, unit, flags, tile index within
+// its unit} (for the end marker: {0, 0, kEntEnd, number of tiles}).  The low
+// two flag bits say which 64-row halves of the query tile attend the key
+// block; bits 8 and up hold the index of the unit among this CTA's units
+// with tiles.
+constexpr int kSchedSlots = 16;  // per ring
+constexpr int kEntFirst = 4;     // first tile of its unit
+constexpr int kEntLast = 8;      // last tile of its unit
+constexpr int kEntEmpty = 16;    // unit without tiles (its output rows are zero)
+constexpr int kEntEnd = 32;      // no more units for this CTA
+constexpr int kEntUnitShift = 8;
+constexpr int kMmaRing = 2;  // ring of the two MMA threads
 
 __device__ __forceinline__ float ex2_approx(float x) {
   float y;
@@ -285,7 +292,7 @@ __device__ __forceinline__ void decode_unit(const AttnParams& p, int u, int& b, 
 template <int RK, int RV>
 struct SharedState {
   uint64_t k_full[RK], k_empty[RK], v_full[RV], v_empty[RV];
-  uint64_t sched_full[kSchedSlots], sched_empty[kSchedSlots];
+  uint64_t sched_full[3][kSchedSlots], sched_empty[3][kSchedSlots];
   // A parity wait is exact only while the barrier is at most one phase away
   // from the awaited one.  Barriers whose waiters may arrive late (after the
   // next phase could complete) or early (before the previous phase has
@@ -299,15 +306,15 @@ struct SharedState {
   uint64_t s_free[2];     // S buffer b read by its softmax warpgroup (4 warps)
   uint64_t p_full[2];     // P(j) written, j & 1 == b (4 warps of warpgroup b)
   uint64_t o_full[2];     // P V(j) completed, j & 1 == b (P V thread commit); also frees P
-  uint64_t o_free;        // both epilogue halves read O (8 softmax warps)
+  uint64_t o_free;        // the epilogue read O (4 warps of L)
   uint64_t m_pub[2][2];   // warpgroup w published its running max, slot = its tile count & 1
-  uint64_t l_pub[2];      // warpgroup w published its row-sum part of a unit
-  uint64_t l_ack[2];      // the other warpgroup read that part
+  uint64_t l_pub[2];      // warpgroup w, as E, published its row-sum part of a unit
+  uint64_t l_ack[2];      // the other warpgroup (L) read that part
   uint64_t epi[2];        // the 4 warps of warpgroup w wrote their block-mass sums
   uint64_t s_done, pv_done;
-  int4 sched[kSchedSlots];
+  int4 sched[3][kSchedSlots];
   float mx[2][2][128];   // [warpgroup][slot][row] running max after a tile
-  float lx[2][128];      // [warpgroup][row] row-sum part at the end of a unit
+  float lx[2][128];      // [warpgroup][row] E's row-sum part at the end of a unit
   float lm[2][128];      // [warpgroup][row] the max that part refers to
   uint32_t tmem_base;
   int abort;
@@ -334,14 +341,20 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
   uint8_t* k_ring = ring;
   uint8_t* v_ring = ring + RK * C::kKVBytes;
   volatile int* abort = &sb.abort;
-  int e = 0, jk = 0, jv = 0, nq = 0, bad = 0;
+  int jk = 0, jv = 0, nq = 0, bad = 0;
+  int jt = 0, n_empty = 0;  // tiles and units without tiles scheduled so far
   bool ok = true;
-  auto emit = [&](int kb, int u, int flags) -> bool {
+  // Writes the next entry of a ring.  Its position follows from the counts:
+  // the MMA ring holds every tile, ring 1 the odd tiles, ring 0 the even
+  // tiles and the units without tiles.
+  auto emit = [&](int ring_w, int kb, int u, int flags, int t) -> bool {
+    const int e = ring_w == kMmaRing ? jt : ring_w == 1 ? (jt >> 1) : ((jt + 1) >> 1) + n_empty;
     const int slot = e % kSchedSlots;
-    if (e >= kSchedSlots && !mbar_wait(&sb.sched_empty[slot], ((e / kSchedSlots) - 1) & 1, abort)) return false;
-    sb.sched[slot] = make_int4(kb, u, flags, 0);
-    mbar_arrive(&sb.sched_full[slot]);  // release: the entry is visible to whoever acquires the phase
-    ++e;
+    if (e >= kSchedSlots &&
+        !mbar_wait(&sb.sched_empty[ring_w][slot], ((e / kSchedSlots) - 1) & 1, abort))
+      return false;
+    sb.sched[ring_w][slot] = make_int4(kb, u, flags, t);
+    mbar_arrive(&sb.sched_full[ring_w][slot]);  // release: the entry is visible to whoever acquires the phase
     return true;
   };
   auto load = [&](const CUtensorMap* map, uint8_t* base, uint64_t* full, uint64_t* empty, int R, int& j, int kb,
@@ -367,15 +380,21 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
     auto it = make_iter<BN, MODE>(p, b, kvh, qt);
     int kb, bits;
     bool have = it.next(kb, bits);
-    if (!have && !emit(0, u, kEntEmpty)) ok = false;
+    if (!have) {
+      if (!emit(0, 0, u, kEntEmpty, 0)) ok = false;
+      ++n_empty;
+    }
     bool first = true;
-    while (have && ok) {
+    const int unit_ix = nq;  // index of this unit among the units with tiles
+    for (int t = 0; have && ok; ++t) {
       int nkb, nbits;
       const bool more = it.next(nkb, nbits);
-      if (!emit(kb, u, bits | (first ? kEntFirst : 0) | (more ? 0 : kEntLast))) {
+      const int flags = bits | (first ? kEntFirst : 0) | (more ? 0 : kEntLast) | (unit_ix << kEntUnitShift);
+      if (!emit(kMmaRing, kb, u, flags, t) || !emit(jt & 1, kb, u, flags, t)) {
         ok = false;
         break;
       }
+      ++jt;
       if (first) {
         // The staging buffer is free once the previous unit's Q is in TMEM.
         if (nq >= 1 && !mbar_wait(&sb.q_stage_free, (nq - 1) & 1, abort)) {
@@ -406,7 +425,8 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
     bad |= it.bad;
   }
   if (ok && have_prev && !load(mapV, v_ring, sb.v_full, sb.v_empty, RV, jv, prev_kb, prev_z)) ok = false;
-  if (ok && !emit(0, 0, kEntEnd)) ok = false;
+  for (int rw = 0; rw < 3 && ok; ++rw)
+    if (!emit(rw, 0, 0, kEntEnd, jt)) ok = false;
   if (bad) atomicOr(p.status, kStatusBadSupport);
   if (!ok) {
     raise_status(p, &sb.abort, kStatusTimeout);
@@ -419,13 +439,13 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
   }
 }
 
-// Reads schedule entry e (single thread).
+// Single thread: reads entry e of the MMA ring (tile e, or the end marker).
 template <class SS>
-__device__ __forceinline__ bool sched_read(SS& sb, int e, int4& ent, volatile int* abort) {
+__device__ __forceinline__ bool sched_read_mma(SS& sb, int e, int4& ent, volatile int* abort) {
   const int slot = e % kSchedSlots;
-  if (!mbar_wait(&sb.sched_full[slot], (e / kSchedSlots) & 1, abort)) return false;
-  ent = sb.sched[slot];
-  mbar_arrive(&sb.sched_empty[slot]);
+  if (!mbar_wait(&sb.sched_full[kMmaRing][slot], (e / kSchedSlots) & 1, abort)) return false;
+  ent = sb.sched[kMmaRing][slot];
+  mbar_arrive(&sb.sched_empty[kMmaRing][slot]);
   return true;
 }
 
@@ -439,14 +459,13 @@ __device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* q_stage,
   constexpr uint32_t idesc_s = idesc_bf16_f32(128, BN, false, false);
   int j = 0, nq = 0;
   bool ok = true;
-  for (int e = 0;; ++e) {
+  for (;;) {
     int4 ent;
-    if (!sched_read(sb, e, ent, abort)) {
+    if (!sched_read_mma(sb, j, ent, abort)) {
       ok = false;
       break;
     }
     if (ent.z & kEntEnd) break;
-    if (ent.z & kEntEmpty) continue;
     if (ent.z & kEntFirst) {
       // Q in TMEM was last read by the S products of unit nq - 1.
       if (nq >= 1 && !mbar_wait(&sb.q_free, (nq - 1) & 1, abort)) {
@@ -508,14 +527,13 @@ __device__ void attn_mma_pv(const AttnParams& p, uint32_t tmem, uint8_t* ring,
   constexpr uint32_t idesc_o = idesc_bf16_f32(128, D, false, true);
   int j = 0, nu = 0;
   bool ok = true;
-  for (int e = 0;; ++e) {
+  for (;;) {
     int4 ent;
-    if (!sched_read(sb, e, ent, abort)) {
+    if (!sched_read_mma(sb, j, ent, abort)) {
       ok = false;
       break;
     }
     if (ent.z & kEntEnd) break;
-    if (ent.z & kEntEmpty) continue;
     const bool first = (ent.z & kEntFirst) != 0;
     if (first) {
       // The first P V of a unit overwrites O: both epilogue halves of the
@@ -552,34 +570,33 @@ __device__ void attn_mma_pv(const AttnParams& p, uint32_t tmem, uint8_t* ring,
   mbar_wait(&sb.pv_done, 0, &never);
 }
 
-// Loads this thread's row of an S tile (kCols columns, one wait) and applies
-// the causal / support masks.
-template <int kCols>
-__device__ __forceinline__ void load_s_row(uint32_t addr, float (&s)[kCols], bool attend, int lim) {
-  static_assert(kCols == 64 || kCols == 128, "tile width");
-  uint32_t va[32], vb[32];
+// Loads N consecutive 32-bit TMEM columns of this thread's lane (N = 64, 96
+// or 128: 32-column loads issued together, one wait).
+template <int N>
+__device__ __forceinline__ void tmem_load_row(uint32_t addr, float (&x)[N]) {
+  static_assert(N == 64 || N == 96 || N == 128, "row width");
+  uint32_t va[32], vb[32], vc[32], vd[32];
   tmem_ld_32x32b_x32(addr, va);
   tmem_ld_32x32b_x32(addr + 32, vb);
-  if constexpr (kCols == 128) {
-    uint32_t vc[32], vd[32];
-    tmem_ld_32x32b_x32(addr + 64, vc);
-    tmem_ld_32x32b_x32(addr + 96, vd);
-    tmem_ld_wait(va, vb);  // completes all four loads
-    reg_tie(vc);
-    reg_tie(vd);
-#pragma unroll
-    for (int e = 0; e < 32; ++e) {
-      s[64 + e] = __uint_as_float(vc[e]);
-      s[96 + e] = __uint_as_float(vd[e]);
-    }
-  } else {
-    tmem_ld_wait(va, vb);
-  }
+  if constexpr (N >= 96) tmem_ld_32x32b_x32(addr + 64, vc);
+  if constexpr (N == 128) tmem_ld_32x32b_x32(addr + 96, vd);
+  tmem_ld_wait(va, vb);  // completes every load issued above
+  if constexpr (N >= 96) reg_tie(vc);
+  if constexpr (N == 128) reg_tie(vd);
 #pragma unroll
   for (int e = 0; e < 32; ++e) {
-    s[e] = __uint_as_float(va[e]);
-    s[32 + e] = __uint_as_float(vb[e]);
+    x[e] = __uint_as_float(va[e]);
+    x[32 + e] = __uint_as_float(vb[e]);
+    if constexpr (N >= 96) x[64 + e] = __uint_as_float(vc[e]);
+    if constexpr (N == 128) x[96 + e] = __uint_as_float(vd[e]);
   }
+}
+
+// Loads this thread's row of an S tile (kCols columns) and applies the
+// causal / support masks.
+template <int kCols>
+__device__ __forceinline__ void load_s_row(uint32_t addr, float (&s)[kCols], bool attend, int lim) {
+  tmem_load_row<kCols>(addr, s);
   // Keys with column c > lim are in the future of this row; a row that does
   // not attend the tile masks every column.
   const int lim_eff = attend ? lim : -1;
@@ -589,22 +606,21 @@ __device__ __forceinline__ void load_s_row(uint32_t addr, float (&s)[kCols], boo
   }
 }
 
-// What an epilogue half needs about its unit.
+// What the epilogue needs about its unit.
 struct EpiInfo {
   int u;      // unit
   int j0;     // tile counter of its first tile
   int j1;     // tile counter of its last tile
   int nu;     // index among this CTA's units with tiles
   int n_kt;   // key tiles 0..n_kt-1 (dense variants)
-  float l, m; // this warpgroup's row-sum part and the max it refers to
+  float l, m; // L's row-sum part and the max it refers to (the final one)
 };
 
 // ------------------------------------------------------------------- softmax
 template <int D, int BN, int MODE>
-__device__ void attn_softmax(const AttnParams& p, int w, uint32_t tmem,
+__device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w, uint32_t tmem, uint8_t* out_stage,
                              SharedState<AttnCfg<D, BN>::kRingK, AttnCfg<D, BN>::kRingV>& sb) {
   using C = AttnCfg<D, BN>;
-  constexpr int kOHalf = D / 2;               // O columns per epilogue half
   constexpr float kRescaleThreshold = 8.0f;   // log2 units: P stays <= 256
   volatile int* abort = &sb.abort;
   const int r = threadIdx.x & 127;  // query row within the tile (TMEM lane)
@@ -613,23 +629,28 @@ __device__ void attn_softmax(const AttnParams& p, int w, uint32_t tmem,
   const uint32_t s_col = C::kTmemS + w * C::kTmemSCols;  // this warpgroup's S buffer
   const uint32_t p_col = C::kTmemP;
   const int half_bit = (BN == 64) ? (1 << (r >> 6)) : 1;
-  // Per-CTA scratch (kDenseMass): this warpgroup's log2 partial masses
-  // [2 units][n_blocks / 2 + 1 tiles][128 rows] (tile t of a unit sits at
-  // t / 2), then [2 warpgroups][2][4 warps][n_blocks] per-warp column sums.
+  // Per-CTA scratch (kDenseMass): log2 partial masses [2 warpgroups][2 units]
+  // [n_blocks / 2 + 1 tiles][128 rows] (tile t of a unit sits at t / 2 in
+  // the region of the warpgroup that handled it), then [2 warpgroups][2]
+  // [4 warps][n_blocks] per-warp column sums.
   const int lc_tiles = p.n_blocks / 2 + 1;
   float* cta_scratch = p.scratch + (size_t)blockIdx.x * scratch_floats_per_cta(p.n_blocks);
-  float* lc_own = cta_scratch + (size_t)w * 2 * lc_tiles * 128;
+  auto lc_at = [&](int g, int unit, int t) -> float* {
+    return cta_scratch + ((size_t)(g * 2 + (unit & 1)) * lc_tiles + (t >> 1)) * 128 + r;
+  };
   float* warp_sums = cta_scratch + (size_t)4 * lc_tiles * 128;
 
-  int j = 0, nu = 0, n_epi = 0;
-  int cur_u = 0, cur_j0 = 0, cur_row = 0;
+  int j = w;             // this warpgroup's next tile: w, w + 2, ...
+  int pos = 0;           // entries read from ring w
+  int n_epi = 0;         // epilogues run (as L); also the other warpgroup's publications read
+  int n_pub = 0;         // publications as E
+  bool fresh = true;     // the row-sum state holds no tile of the current unit
+  int cur_row = 0;
   float l_w = 0.0f, m_w = -INFINITY;  // this warpgroup's part of the row sum, relative to m_w
-  bool pend = false;
-  EpiInfo pe{};
   bool ok = true;
 
-  // ---- one tile (j & 1 == w)
-  auto tile = [&](int kb, int bits, bool first) -> bool {
+  // ---- one tile (j & 1 == w): key block kb, tile t of the unit with index unit_ix
+  auto tile = [&](int kb, int bits, bool first, int t, int unit_ix) -> bool {
     if (!warp_wait(&sb.s_full[w], (j >> 1) & 1, abort)) return false;
     tc_fence_after_sync();
     const bool attend = (bits & half_bit) != 0;
@@ -672,9 +693,11 @@ __device__ void attn_softmax(const AttnParams& p, int w, uint32_t tmem,
       m_w = m_new;
     }
     l_w += rowsum;
-    if (MODE == kDenseMass)
-      lc_own[((size_t)(nu & 1) * lc_tiles + ((j - cur_j0) >> 1)) * 128 + r] =
-          rowsum > 0.0f ? m_new + lg2_approx(rowsum) : -INFINITY;
+    // Written after the P V(j-1) wait above: tile j-1 was handled by the
+    // other warpgroup after any epilogue it ran for unit unit_ix - 2 (which
+    // read this slot), and this warpgroup's own epilogues precede in program
+    // order.
+    if (MODE == kDenseMass) *lc_at(w, unit_ix, t) = rowsum > 0.0f ? m_new + lg2_approx(rowsum) : -INFINITY;
     // O (after P V(j-1)) is rescaled only when the max moved.  tcgen05.ld/st
     // are warp-collective: the warp rescales together, lanes whose max did
     // not move use a factor of 1.
@@ -698,55 +721,62 @@ __device__ void attn_softmax(const AttnParams& p, int w, uint32_t tmem,
     return true;
   };
 
-  // ---- this warpgroup's half of a unit's epilogue
+  // ---- the epilogue, run by L (this warpgroup handled the unit's last tile)
   auto epilogue = [&](const EpiInfo& ei) -> bool {
-    const int x = w ^ 1;
-    if (!warp_wait(&sb.l_pub[x], ei.nu & 1, abort)) return false;
-    const float l_o = sb.lx[x][r], m_o = sb.lm[x][r];
+    const int x = w ^ 1;  // E
+    if (!warp_wait(&sb.l_pub[x], n_epi & 1, abort)) return false;
+    const float lE = sb.lx[x][r], mE = sb.lm[x][r];
     __syncwarp();
     if (lane == 0) mbar_arrive(&sb.l_ack[x]);
-    // L handled the last tile: its max is the one O refers to, and E's max
-    // is at most that.
-    const bool is_L = ((ei.j1 & 1) == w);
-    const float lL = is_L ? ei.l : l_o, mL = is_L ? ei.m : m_o;
-    const float lE = is_L ? l_o : ei.l, mE = is_L ? m_o : ei.m;
-    const float l_row = (mE == -INFINITY) ? lL : lL + lE * ex2_approx(mE - mL);
-    // P V(j1-2) completed before P(j1) was written, which the other part
-    // published above presupposes (or this warpgroup's tile j1 itself).
+    // O refers to L's max, which is the final running max; E's is at most
+    // that.
+    const float l_row = (mE == -INFINITY) ? ei.l : ei.l + lE * ex2_approx(mE - ei.m);
+    // P V(j1-1) completed before P(j1) was written, so o_full[j1 & 1] is at
+    // most one phase short of P V(j1).
     if (!warp_wait(&sb.o_full[ei.j1 & 1], (ei.j1 >> 1) & 1, abort)) return false;
     tc_fence_after_sync();
+    float o[D];
+    tmem_load_row<D>(lane_tmem + C::kTmemO, o);
+    tc_fence_before_sync();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&sb.o_free);
     int b, h, qt;
     decode_unit(p, ei.u, b, h, qt);
     const int row = qt * 128 + r;
     const float inv_l = l_row > 0.0f ? 1.0f / l_row : 0.0f;
-    __nv_bfloat16* orow = p.O + ((size_t)(b * p.n_heads + h) * p.seqlen + row) * D + w * kOHalf;
+    // O / l through this warp's staging box (32 rows x 64 columns, 128-byte
+    // swizzle) and a TMA store per 64 columns; rows past seqlen are dropped.
+    uint8_t* stage = out_stage + wq * (32 * 128);
 #pragma unroll
-    for (int c = 0; c < kOHalf / 16; ++c) {
-      uint32_t v[16];
-      tmem_ld_32x32b_x16(lane_tmem + C::kTmemO + w * kOHalf + 16 * c, v);
-      tmem_ld_wait(v);
-      uint32_t o[8];
+    for (int hb = 0; hb < C::kBoxes; ++hb) {
+      // The previous store from the staging box has read it.
+      if (lane == 0) tma_store_wait_read();
+      __syncwarp();
 #pragma unroll
-      for (int e = 0; e < 8; ++e)
-        o[e] = pack_bf16x2(__uint_as_float(v[2 * e]) * inv_l, __uint_as_float(v[2 * e + 1]) * inv_l);
-      if (row < p.seqlen) {
-        uint4* dst = reinterpret_cast<uint4*>(orow + 16 * c);
-        dst[0] = make_uint4(o[0], o[1], o[2], o[3]);
-        dst[1] = make_uint4(o[4], o[5], o[6], o[7]);
+      for (int c = 0; c < 8; ++c) {
+        const int col = hb * 64 + c * 8;
+        uint32_t q[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          q[e] = (col + 2 * e + 1 < D) ? pack_bf16x2(o[col + 2 * e] * inv_l, o[col + 2 * e + 1] * inv_l) : 0u;
+        st_shared_v4(smem_u32(stage + lane * 128 + ((c ^ (lane & 7)) << 4)), q[0], q[1], q[2], q[3]);
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        tma_store_3d(mapO, stage, hb * 64, qt * 128 + wq * 32, b * p.n_heads + h);
+        tma_store_commit();
       }
     }
-    tc_fence_before_sync();
-    __syncwarp();
-    if (lane == 0) mbar_arrive(&sb.o_free);
     if constexpr (MODE == kDenseMass) {
-      // Block mass (Eq. 5) of this warpgroup's tiles: per row
-      // 2^(lc - lse), summed over the rows of each query block.
-      const float lse = mL + lg2_approx(l_row);
+      // Block mass (Eq. 5): per row 2^(lc - lse), summed over the rows of
+      // each query block.  E wrote its tiles' lc before publishing its part.
+      const float lse = ei.m + lg2_approx(l_row);
       float* ws = warp_sums + (size_t)(w * 2 + (n_epi & 1)) * 4 * p.n_blocks;
       const int n_kt = ei.n_kt;
       // Dense variants: tile t of the unit is key block t.
-      for (int t = (w - ei.j0) & 1; t < n_kt; t += 2) {
-        const float lc = lc_own[((size_t)(ei.nu & 1) * lc_tiles + (t >> 1)) * 128 + r];
+      for (int t = 0; t < n_kt; ++t) {
+        const float lc = *lc_at((ei.j0 + t) & 1, ei.nu, t);
         float v = (row < p.seqlen) ? ex2_approx(lc - lse) : 0.0f;
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
@@ -757,15 +787,12 @@ __device__ void attn_softmax(const AttnParams& p, int w, uint32_t tmem,
       __syncwarp();
       if (lane == 0) mbar_arrive(&sb.epi[w]);
       if (!warp_wait(&sb.epi[w], n_epi & 1, abort)) return false;
-      ++n_epi;
       constexpr int kHalves = 128 / BN;  // query blocks per tile
       const float inv_b = 1.0f / (float)BN;
       for (int e = r; e < kHalves * p.n_blocks; e += 128) {
         const int hf = e / p.n_blocks, t = e % p.n_blocks;
         const int qblock = qt * kHalves + hf;
         if (qblock >= p.n_blocks) continue;
-        const bool own = (t < n_kt) ? (((ei.j0 + t) & 1) == w) : ((t & 1) == w);
-        if (!own) continue;
         float* out = p.blockmass + ((size_t)(b * p.n_heads + h) * p.n_blocks + qblock) * p.n_blocks + t;
         if (t < n_kt) {
           float sum = 0.0f;
@@ -783,82 +810,86 @@ __device__ void attn_softmax(const AttnParams& p, int w, uint32_t tmem,
         }
       }
     }
+    ++n_epi;
     return true;
   };
 
-  for (int e = 0; ok; ++e) {
-    const int slot = e % kSchedSlots;
-    if (!warp_wait(&sb.sched_full[slot], (e / kSchedSlots) & 1, abort)) {
+  // ---- E's publication of its part of the row sum for the unit that just
+  // ended (zero if this warpgroup handled none of its tiles), once L has read
+  // the previous one.
+  auto publish = [&]() -> bool {
+    if (n_pub >= 1 && !warp_wait(&sb.l_ack[w], (n_pub - 1) & 1, abort)) return false;
+    sb.lx[w][r] = fresh ? 0.0f : l_w;
+    sb.lm[w][r] = fresh ? -INFINITY : m_w;
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&sb.l_pub[w]);
+    ++n_pub;
+    fresh = true;
+    return true;
+  };
+
+  for (;;) {
+    const int slot = pos % kSchedSlots;
+    if (!warp_wait(&sb.sched_full[w][slot], (pos / kSchedSlots) & 1, abort)) {
       ok = false;
       break;
     }
-    const int4 ent = sb.sched[slot];
+    const int4 ent = sb.sched[w][slot];
     __syncwarp();
-    if (lane == 0) mbar_arrive(&sb.sched_empty[slot]);
+    if (lane == 0) mbar_arrive(&sb.sched_empty[w][slot]);
+    ++pos;
     const int fl = ent.z;
-    if (fl & kEntEnd) break;
+    if (fl & kEntEnd) {
+      // The last unit ended at tile ent.w - 1; if the other warpgroup handled
+      // it, this one is that unit's E.
+      if (ent.w >= 1 && ((ent.w - 1) & 1) != w && !publish()) ok = false;
+      break;
+    }
     if (fl & kEntEmpty) {
-      // No key tile: the rows of the unit attend nothing and are zero.
+      // No key tile (ring 0 only): the rows of the unit attend nothing and
+      // are zero.
       int b, h, qt;
       decode_unit(p, ent.y, b, h, qt);
       const int row = qt * 128 + r;
       if (row < p.seqlen) {
-        uint4* dst = reinterpret_cast<uint4*>(p.O + ((size_t)(b * p.n_heads + h) * p.seqlen + row) * D + w * kOHalf);
+        uint4* dst = reinterpret_cast<uint4*>(p.O + ((size_t)(b * p.n_heads + h) * p.seqlen + row) * D);
 #pragma unroll
-        for (int c = 0; c < kOHalf / 8; ++c) dst[c] = make_uint4(0u, 0u, 0u, 0u);
+        for (int c = 0; c < D / 8; ++c) dst[c] = make_uint4(0u, 0u, 0u, 0u);
       }
       continue;
     }
-    if (fl & kEntFirst) {
+    const bool first = (fl & kEntFirst) != 0;
+    // Tile j - 1 (the other warpgroup's) ended the previous unit: this
+    // warpgroup is that unit's E.
+    if (first && j >= 1 && !publish()) {
+      ok = false;
+      break;
+    }
+    if (fresh) {
       int b, h, qt;
       decode_unit(p, ent.y, b, h, qt);
-      cur_u = ent.y;
-      cur_j0 = j;
       cur_row = qt * 128 + r;
       l_w = 0.0f;
       m_w = -INFINITY;
     }
-    if ((j & 1) == w) {
-      if (!tile(ent.x, fl & 3, (fl & kEntFirst) != 0)) {
-        ok = false;
-        break;
-      }
-      // A deferred epilogue half runs after this warpgroup's first tile of
-      // the following unit.
-      if (pend) {
-        if (!epilogue(pe)) {
-          ok = false;
-          break;
-        }
-        pend = false;
-      }
+    if (!tile(ent.x, fl & 3, first, ent.w, fl >> kEntUnitShift)) {
+      ok = false;
+      break;
     }
+    fresh = false;
     if (fl & kEntLast) {
-      // Publish this warpgroup's part of the row sum (once the other one has
-      // read the previous unit's part).
-      if (nu >= 1 && !warp_wait(&sb.l_ack[w], (nu - 1) & 1, abort)) {
+      // L: this warpgroup handled the unit's last tile.
+      const EpiInfo ei{ent.y, j - ent.w, j, fl >> kEntUnitShift, ent.x + 1, l_w, m_w};
+      if (!epilogue(ei)) {
         ok = false;
         break;
       }
-      sb.lx[w][r] = l_w;
-      sb.lm[w][r] = m_w;
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&sb.l_pub[w]);
-      const EpiInfo ei{cur_u, cur_j0, j, nu, ent.x + 1, l_w, m_w};
-      ++nu;
-      if ((j & 1) == w) {
-        if (!epilogue(ei)) {
-          ok = false;
-          break;
-        }
-      } else {
-        pe = ei;
-        pend = true;
-      }
+      fresh = true;
     }
-    ++j;
+    j += 2;
   }
-  if (ok && pend) ok = epilogue(pe);
+  // Output stores issued by this warp must complete before the CTA exits.
+  if (lane == 0) tma_store_wait_all();
   if (!ok) raise_status(p, &sb.abort, kStatusTimeout);
 }
 
@@ -866,7 +897,8 @@ __device__ void attn_softmax(const AttnParams& p, int w, uint32_t tmem,
 template <int D, int BN, int MODE>
 __global__ void __launch_bounds__(AttnCfg<D, BN>::kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
-                const __grid_constant__ CUtensorMap mapV, const AttnParams p) {
+                const __grid_constant__ CUtensorMap mapV, const __grid_constant__ CUtensorMap mapO,
+                const AttnParams p) {
   using C = AttnCfg<D, BN>;
   using SS = SharedState<C::kRingK, C::kRingV>;
   static_assert(sizeof(SS) <= C::kStaticReserve, "static shared memory");
@@ -874,6 +906,7 @@ __global__ void __launch_bounds__(AttnCfg<D, BN>::kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* q_stage = smem;             // one Q tile
   uint8_t* ring = smem + C::kQBytes;   // kRing K/V entries
+  uint8_t* out_stage = ring + C::kRing * C::kKVBytes;  // epilogue staging (1024-byte aligned)
   __shared__ SS sb;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -888,8 +921,10 @@ __global__ void __launch_bounds__(AttnCfg<D, BN>::kThreads, 1)
       mbar_init(&sb.v_empty[i], 1);
     }
     for (int i = 0; i < kSchedSlots; ++i) {
-      mbar_init(&sb.sched_full[i], 1);
-      mbar_init(&sb.sched_empty[i], kSchedReaders);
+      for (int rw = 0; rw < 3; ++rw) {
+        mbar_init(&sb.sched_full[rw][i], 1);
+        mbar_init(&sb.sched_empty[rw][i], rw == kMmaRing ? 2 : 4);  // its readers
+      }
     }
     mbar_init(&sb.q_full, 1);
     mbar_init(&sb.q_stage_free, 1);
@@ -905,7 +940,7 @@ __global__ void __launch_bounds__(AttnCfg<D, BN>::kThreads, 1)
       mbar_init(&sb.epi[b], 4);
       mbar_init(&sb.o_full[b], 1);
     }
-    mbar_init(&sb.o_free, 8);
+    mbar_init(&sb.o_free, 4);
     mbar_init(&sb.s_done, 1);
     mbar_init(&sb.pv_done, 1);
     fence_mbar_init();
@@ -914,6 +949,7 @@ __global__ void __launch_bounds__(AttnCfg<D, BN>::kThreads, 1)
     tma_prefetch_map(&mapQ);
     tma_prefetch_map(&mapK);
     tma_prefetch_map(&mapV);
+    tma_prefetch_map(&mapO);
   }
   if (warp == C::kMmaSWarp) {
     tmem_alloc(&sb.tmem_base, C::kTmemCols);
@@ -926,7 +962,7 @@ __global__ void __launch_bounds__(AttnCfg<D, BN>::kThreads, 1)
 
   if (warp < 8) {
     warpgroup_reg_inc<C::kRegsSoftmax>();
-    attn_softmax<D, BN, MODE>(p, warp >> 2, tmem, sb);
+    attn_softmax<D, BN, MODE>(&mapO, p, warp >> 2, tmem, out_stage, sb);
   } else {
     warpgroup_reg_dec<C::kRegsOther>();
     if (warp == C::kProducerWarp) {
@@ -954,7 +990,7 @@ cudaError_t launch_attn_instance(const AttnLaunch& L) {
   auto kern = attn_kernel<D, BN, MODE>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemLaunch);
   if (e != cudaSuccess) return e;
-  kern<<<L.grid, C::kThreads, C::kSmemLaunch, L.stream>>>(L.mapQ, L.mapK, L.mapV, L.p);
+  kern<<<L.grid, C::kThreads, C::kSmemLaunch, L.stream>>>(L.mapQ, L.mapK, L.mapV, L.mapO, L.p);
   return cudaGetLastError();
 }
 

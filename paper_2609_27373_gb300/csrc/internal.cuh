@@ -43,6 +43,7 @@ struct AttnParams {
 
 struct AttnLaunch {
   CUtensorMap mapQ, mapK, mapV;
+  CUtensorMap mapO;  // output, 32-row boxes (TMA stores of the epilogue)
   AttnParams p;
   int grid;
   cudaStream_t stream;

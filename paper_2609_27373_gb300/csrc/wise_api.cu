@@ -110,7 +110,8 @@ int check_shape(const wise_shape_t* sh, bool attention) {
 }
 
 // Tensor map over a [rows_outer, seqlen, head_dim] bf16 array with 64-column,
-// box_rows-row boxes in the 128-byte swizzle.  Rows past seqlen read as zero.
+// box_rows-row boxes in the 128-byte swizzle.  Rows past seqlen read as zero
+// and are not written by stores.
 bool make_map(CUtensorMap* map, const void* base, int head_dim, int seqlen, long long outer, int box_rows) {
   EncodeTiledFn enc = encode_tiled();
   if (!enc) return false;
@@ -149,7 +150,8 @@ int launch_attention(const wise_shape_t* sh, const void* Q, const void* K, const
   const long long outer_kv = (long long)sh->batch * sh->n_kv_heads;
   if (!make_map(&L.mapQ, Q, sh->head_dim, sh->seqlen, outer_q, 128) ||
       !make_map(&L.mapK, K, sh->head_dim, sh->seqlen, outer_kv, sh->block) ||
-      !make_map(&L.mapV, V, sh->head_dim, sh->seqlen, outer_kv, sh->block))
+      !make_map(&L.mapV, V, sh->head_dim, sh->seqlen, outer_kv, sh->block) ||
+      !make_map(&L.mapO, O, sh->head_dim, sh->seqlen, outer_q, 32))
     return WISE_ERR_CUDA;
 
   AttnParams& p = L.p;
