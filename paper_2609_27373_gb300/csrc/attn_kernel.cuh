@@ -674,19 +674,23 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     __syncwarp();
     if (lane == 0) mbar_arrive(&sb.m_pub[w][(j >> 1) & 1]);
     const float rowsum = exp2_scaled(s, p.scale_log2, m_new == -INFINITY ? 0.0f : m_new);
+    // P as bf16 pairs, packed before the wait below.
+    uint32_t pw[BN / 2];
+#pragma unroll
+    for (int e = 0; e < BN / 2; ++e) pw[e] = pack_bf16x2(s[2 * e], s[2 * e + 1]);
     // P was last read by P V(j-1), and O must have received it before a
     // rescale.  P V(j-2) completed before tile j-1's P was written, which this
     // warpgroup's own previous wait (or the exchange of the running max)
     // implies, so o_full[(j-1) & 1] is at most one phase short of P V(j-1).
     if (j >= 1 && !warp_wait(&sb.o_full[(j - 1) & 1], ((j - 1) >> 1) & 1, abort)) return false;
     tc_fence_after_sync();
-    // P as bf16 pairs; the stores complete while the bookkeeping below runs.
+    // The stores complete while the bookkeeping below runs.
 #pragma unroll
     for (int c = 0; c < BN / 32; ++c) {
-      uint32_t pw[16];
+      uint32_t q[16];
 #pragma unroll
-      for (int e = 0; e < 16; ++e) pw[e] = pack_bf16x2(s[32 * c + 2 * e], s[32 * c + 2 * e + 1]);
-      tmem_st_32x32b_x16(lane_tmem + p_col + 16 * c, pw);
+      for (int e = 0; e < 16; ++e) q[e] = pw[16 * c + e];
+      tmem_st_32x32b_x16(lane_tmem + p_col + 16 * c, q);
     }
     if (m_new != m_w) {
       l_w *= ex2_approx(m_w - m_new);  // 0 while m_w is -inf
