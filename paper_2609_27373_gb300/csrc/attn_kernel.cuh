@@ -23,12 +23,14 @@
 //                shared memory (K-major);
 //   O += P V     P written by the softmax into TMEM, V from shared memory
 //                (MN-major).
-// TMEM (512 columns): Q (64 columns), P (64 columns), S double-buffered
-// across tiles (2 x 128 columns), O (128 columns).  S(j+2) is issued as soon
-// as the softmax has read S(j) into registers, so the S product runs up to two
-// tiles ahead and never waits for a P V; P(j) waits for P V(j-1), which
-// normally completed while the softmax of tile j ran.  The Q of the next unit
-// is copied in once the last S product of the current unit has completed.
+// TMEM (512 columns, 448 used): Q (64 columns), one S buffer (128 columns), P
+// double-buffered across tiles (2 x 64 columns), O (128 columns).  S(j+1) is
+// issued as soon as the softmax has read S(j) into registers, so the S product
+// never waits for a P V, and P(j) waits only for P V(j-2).  (With two S
+// buffers and one P buffer instead, P(j) has to wait for P V(j-1), which may
+// sit behind an S product in the tensor pipe: a serial P -> P V -> P chain
+// that measured slower.)  The Q of the next unit is copied in once the last S
+// product of the current unit has completed.
 //
 // Warp roles (384 threads; warp 11 only completes warpgroup 2):
 //   warp 8     producer.  Walks the CTA's units, validates the support lists,
@@ -40,13 +42,13 @@
 //              TMA loads of Q (staging buffer), K (ring of kRingK) and V (ring
 //              of kRingV) in the order Q, K(0), K(1), V(0), K(2), V(1), ...
 //   warp 9     S issuer: copies each unit's Q into TMEM and issues
-//              S(j) = Q K(j)^T into S buffer j & 1 once S(j-2) has been read.
+//              S(j) = Q K(j)^T once S(j-1) has been read.
 //   warp 10    P V issuer: O += P(j) V(j) once the softmax has written P(j).
 //              A tcgen05.mma issue blocks its thread while the tensor core
 //              drains earlier instructions, so the two products are issued
 //              from two threads.
 //   warps 0-3 and 4-7  softmax warpgroups 0 and 1.  Warpgroup w handles the
-//              tiles j with j & 1 == w (so it always reads S buffer w); thread
+//              tiles j with j & 1 == w (so it always writes P buffer w); thread
 //              t of a warpgroup owns query row t (= TMEM lane t) and the whole
 //              row of each of its tiles.  The online softmax runs in the log2
 //              domain with one running max m per row shared by both
@@ -98,9 +100,9 @@ struct AttnCfg {
   // TMEM columns).
   static constexpr int kSmemLaunch = kSmemBytes > 116 * 1024 ? kSmemBytes : 116 * 1024;
   static constexpr uint32_t kTmemQ = 0;       // Q: 128 bf16 per row
-  static constexpr uint32_t kTmemP = 64;      // P: 128 bf16 per row
-  static constexpr uint32_t kTmemS = 128;     // two S buffers
-  static constexpr uint32_t kTmemSCols = 128;
+  static constexpr uint32_t kTmemS = 128;     // one S buffer
+  static constexpr uint32_t kTmemP = 256;     // two P buffers of 64 columns
+  static constexpr uint32_t kTmemPCols = 64;
   static constexpr uint32_t kTmemO = 384;     // O accumulator
   static constexpr uint32_t kTmemCols = 512;
   // Warps 0-7 softmax, 8 producer, 9 and 10 MMA issuers, 11 idle (it
@@ -302,10 +304,10 @@ struct SharedState {
   uint64_t q_full;        // Q tile landed in the staging buffer (TMA)
   uint64_t q_stage_free;  // staging buffer copied into TMEM (S thread commit)
   uint64_t q_free;        // last S of a unit completed (S thread commit)
-  uint64_t s_full[2];     // S buffer b written (S thread commit)
-  uint64_t s_free[2];     // S buffer b read by its softmax warpgroup (4 warps)
+  uint64_t s_full[2];     // S(j) written, j & 1 == b (S thread commit)
+  uint64_t s_free[2];     // S(j) read by its softmax warpgroup, j & 1 == b (4 warps)
   uint64_t p_full[2];     // P(j) written, j & 1 == b (4 warps of warpgroup b)
-  uint64_t o_full[2];     // P V(j) completed, j & 1 == b (P V thread commit); also frees P
+  uint64_t o_full[2];     // P V(j) completed, j & 1 == b (P V thread commit); frees P buffer b
   uint64_t o_free;        // the epilogue read O (4 warps of L)
   uint64_t m_pub[2][2];   // warpgroup w published its running max, slot = its tile count & 1
   uint64_t l_pub[2];      // warpgroup w, as E, published its row-sum part of a unit
@@ -490,13 +492,13 @@ __device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* q_stage,
       ok = false;
       break;
     }
-    // S(j) overwrites S(j-2): its softmax warpgroup must have read it.
-    if (j >= 2 && !mbar_wait(&sb.s_free[j & 1], ((j >> 1) - 1) & 1, abort)) {
+    // S(j) overwrites S(j-1): its softmax warpgroup must have read it.
+    if (j >= 1 && !mbar_wait(&sb.s_free[(j - 1) & 1], ((j - 1) >> 1) & 1, abort)) {
       ok = false;
       break;
     }
     tc_fence_after_sync();
-    const uint32_t s_col = C::kTmemS + (j & 1) * C::kTmemSCols;
+    const uint32_t s_col = C::kTmemS;
     const uint64_t b0 = smem_desc_sw128(smem_u32(ring + slot * C::kKVBytes), 16, 1024);
 #pragma unroll 1
     for (int kk = 0; kk < D / 16; ++kk) {
@@ -554,7 +556,7 @@ __device__ void attn_mma_pv(const AttnParams& p, uint32_t tmem, uint8_t* ring,
       break;
     }
     tc_fence_after_sync();
-    const uint32_t p_col = C::kTmemP;
+    const uint32_t p_col = C::kTmemP + (j & 1) * C::kTmemPCols;
     const uint64_t b0 = smem_desc_sw128(smem_u32(v_ring + slot * C::kKVBytes), BN * 128, 1024);
 #pragma unroll 1
     for (int kk = 0; kk < BN / 16; ++kk)
@@ -626,8 +628,8 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
   const int r = threadIdx.x & 127;  // query row within the tile (TMEM lane)
   const int wq = r >> 5, lane = r & 31;
   const uint32_t lane_tmem = tmem + ((uint32_t)(wq * 32) << 16);
-  const uint32_t s_col = C::kTmemS + w * C::kTmemSCols;  // this warpgroup's S buffer
-  const uint32_t p_col = C::kTmemP;
+  const uint32_t s_col = C::kTmemS;
+  const uint32_t p_col = C::kTmemP + w * C::kTmemPCols;  // this warpgroup's P buffer
   const int half_bit = (BN == 64) ? (1 << (r >> 6)) : 1;
   // Per-CTA scratch (kDenseMass): log2 partial masses [2 warpgroups][2 units]
   // [n_blocks / 2 + 1 tiles][128 rows] (tile t of a unit sits at t / 2 in
@@ -657,7 +659,7 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     const int lim = cur_row - kb * BN;  // keys kb*BN + c with c > lim are in the future
     float s[BN];
     load_s_row<BN>(lane_tmem + s_col, s, attend, lim);
-    // S(j) is in registers: S(j+2) may overwrite it.
+    // S(j) is in registers: S(j+1) may overwrite it.
     tc_fence_before_sync();
     __syncwarp();
     if (lane == 0) mbar_arrive(&sb.s_free[w]);
@@ -678,11 +680,9 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     uint32_t pw[BN / 2];
 #pragma unroll
     for (int e = 0; e < BN / 2; ++e) pw[e] = pack_bf16x2(s[2 * e], s[2 * e + 1]);
-    // P was last read by P V(j-1), and O must have received it before a
-    // rescale.  P V(j-2) completed before tile j-1's P was written, which this
-    // warpgroup's own previous wait (or the exchange of the running max)
-    // implies, so o_full[(j-1) & 1] is at most one phase short of P V(j-1).
-    if (j >= 1 && !warp_wait(&sb.o_full[(j - 1) & 1], ((j - 1) >> 1) & 1, abort)) return false;
+    // P buffer w was last read by P V(j-2); this warpgroup waited for P V(j-4)
+    // at its previous tile, so o_full[w] is at most one phase short.
+    if (j >= 2 && !warp_wait(&sb.o_full[w], ((j >> 1) - 1) & 1, abort)) return false;
     tc_fence_after_sync();
     // The stores complete while the bookkeeping below runs.
 #pragma unroll
@@ -707,6 +707,9 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     // not move use a factor of 1.
     const bool rescale = !first && m_new != m_prev && m_prev != -INFINITY;
     if (__any_sync(0xffffffffu, rescale)) {
+      // O must have received P V(j-1); P V(j-3) completed (the wait above).
+      if (!warp_wait(&sb.o_full[(j - 1) & 1], ((j - 1) >> 1) & 1, abort)) return false;
+      tc_fence_after_sync();
       const float f = rescale ? ex2_approx(m_prev - m_new) : 1.0f;
 #pragma unroll
       for (int c = 0; c < D / 16; ++c) {
@@ -735,7 +738,7 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     // O refers to L's max, which is the final running max; E's is at most
     // that.
     const float l_row = (mE == -INFINITY) ? ei.l : ei.l + lE * ex2_approx(mE - ei.m);
-    // P V(j1-1) completed before P(j1) was written, so o_full[j1 & 1] is at
+    // P V(j1-2) completed before P(j1) was written, so o_full[j1 & 1] is at
     // most one phase short of P V(j1).
     if (!warp_wait(&sb.o_full[ei.j1 & 1], (ei.j1 >> 1) & 1, abort)) return false;
     tc_fence_after_sync();
