@@ -364,6 +364,54 @@ def main():
     e_end.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e_start.elapsed_time(e_end) / e2e_iters
+
+    # ---- sparse kernel with every admissible block (the matched-backend row)
+    nb = shape.n_blocks
+    all_idx, all_counts = synth.all_blocks_support(wl.batch, wl.n_kv_heads, nb)
+    all_idx, all_counts = torch.from_numpy(all_idx).cuda(), torch.from_numpy(all_counts).cuda()
+    ab_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_late)]
+    for i, t in enumerate(range(wl.n_discovery, wl.steps)):
+        Q, K, V = dev_steps[t]
+        ab_ev[i][0].record(stream)
+        wise.wise_sparse_attn(shape, Q, K, V, all_idx, all_counts, O)
+        ab_ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    all_blocks_ms = statistics.mean(a.elapsed_time(b) for a, b in ab_ev)
+
+    # ---- routing diagnostic: share of each late step's full attention kept
+    # by the frozen support (the step's own block mass, then the support sum)
+    diag_mass = torch.empty((wl.batch, wl.n_heads, nb, nb), dtype=torch.float32, device="cuda")
+    retained = torch.empty((wl.batch, wl.n_heads, nb), dtype=torch.float32, device="cuda")
+    ret = []
+    for t in range(wl.n_discovery, wl.steps, 4):
+        Q, K, V = dev_steps[t]
+        wise.wise_full_attn_accumulate(shape, Q, K, V, O, diag_mass, 0)
+        wise.wise_support_mass(shape, diag_mass, layer.idx, layer.counts, retained)
+        ret.append(float(retained.mean()))
+    retained_mass = statistics.mean(ret)
+
+    # ---- the whole trajectory as one CUDA graph (discovery, selection, late
+    # steps), replayed; its launches carry no host-side gaps
+    graph = {"ms": None, "note": None}
+    try:
+        for _ in range(2):
+            trajectory()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            trajectory()
+        g.replay()
+        torch.cuda.synchronize()
+        g_start, g_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = max(3, args.steps // 2)
+        g_start.record(stream)
+        for _ in range(reps):
+            g.replay()
+        g_end.record(stream)
+        torch.cuda.synchronize()
+        graph["ms"] = g_start.elapsed_time(g_end) / reps
+    except Exception as exc:  # report, do not fail the bench line
+        graph["note"] = f"capture failed: {type(exc).__name__}: {exc}"[:200]
     clk = clocks.stop()
     status = wise.wise_get_status()
     if status != wise.WISE_OK:
@@ -407,6 +455,12 @@ def main():
         "tflops_effective": round(achieved, 2),
         "dense_tflops": round(flops_dense / (dense * 1e-3) / 1e12, 2),
         "density": round(density, 4),
+        "retained_mass": round(retained_mass, 4),
+        "all_blocks_ms": round(all_blocks_ms, 5),
+        "all_blocks_vs_dense": round(all_blocks_ms / dense, 4),
+        "graph_trajectory_ms": None if graph["ms"] is None else round(graph["ms"], 4),
+        "graph_trajectory_speedup": None if graph["ms"] is None else round(wl.steps * dense / graph["ms"], 4),
+        **({"graph_note": graph["note"]} if graph["note"] else {}),
         "roofline": {"bound": "tensor", "achieved": round(achieved, 2), "peak": peak, "unit": "TFLOP/s",
                      "frac": round(achieved / peak, 4), "traffic": sparse_traffic_bytes(),
                      "peak_kind": f"{peak_kind} bf16 burst", "kernel": "wise_sparse_attn"},

@@ -141,6 +141,22 @@ int wise_full_attn_accumulate_noalloc(const wise_shape_t* shape, const void* Q, 
 int wise_select_support(const wise_shape_t* shape, const wise_select_t* sel, const float* blockmass,
                         int32_t* idx, int32_t* counts, cudaStream_t stream);
 
+/* Routing diagnostic (appendix "Experimental details", evaluation metrics:
+ * retained future attention mass).  For every query-head row (b, h, q):
+ *   retained[b][h][q] = sum over the key blocks kb of the support list of
+ *                       the kv-group of h of blockmass[b][h][q][kb]
+ * With blockmass = one step's mass (wise_full_attn_accumulate with step 0 on
+ * that step's Q, K, V, i.e. Eq. 5 of the unrestricted attention), this is the
+ * fraction of the step's full attention that the frozen support keeps (1 for
+ * a support holding every admissible block).
+ * blockmass: fp32 [batch, n_heads, nQB, nKB]; idx, counts: as produced by
+ * wise_select_support (row width `cap`); retained: fp32 [batch, n_heads, nQB],
+ * written.  The sum is fp32 in list order (deterministic).  List entries that
+ * are negative, beyond the query block, or not strictly ascending are skipped
+ * and reported as WISE_ERR_BAD_SUPPORT by wise_get_status. */
+int wise_support_mass(const wise_shape_t* shape, const float* blockmass, const int32_t* idx, const int32_t* counts,
+                      int cap, float* retained, cudaStream_t stream);
+
 /* Attention of one late recurrent step restricted to the block support
  *   R_ij = 0 if b(j) in B_q(i) else -inf                              (Eq. 7)
  *   O = softmax(Q K^T * scale + M + R) V, M causal                    (Eq. 8)

@@ -151,3 +151,38 @@ def select_support(blockmass, n_kv_heads, block, mode, n_sink, n_local, topk, et
     if rc != 0:
         raise ValueError("oracle select_support rejected its arguments")
     return idx, counts
+
+
+def support_mass(blockmass, idx, counts, n_heads):
+    """Retained mass of a support (appendix "Experimental details",
+    evaluation metrics: the fraction of the unrestricted attention mass that
+    falls inside the frozen support), per query-head row: the row's block
+    masses r_qb (Eq. 5) summed over the key blocks of its kv-group's support
+    list, in fp64.  List entries that are negative, beyond the query block or
+    not strictly above the last accepted entry are skipped, as the attention
+    kernels skip them.
+
+    blockmass [B,H,nQB,nKB]; idx [B,Hkv,nQB,cap]; counts [B,Hkv,nQB].
+    Returns retained [B,H,nQB] float64.
+    """
+    m = np.asarray(blockmass, dtype=np.float64)
+    B, H, nq, _ = m.shape
+    Hkv = idx.shape[1]
+    if H != n_heads or H % Hkv:
+        raise ValueError("head counts do not match")
+    group = H // Hkv
+    out = np.zeros((B, H, nq), dtype=np.float64)
+    for b in range(B):
+        for h in range(H):
+            for q in range(nq):
+                n = int(counts[b, h // group, q])
+                n = min(max(n, 0), idx.shape[3])
+                prev = -1
+                total = 0.0
+                for v in idx[b, h // group, q, :n]:
+                    v = int(v)
+                    if 0 <= v <= q and v > prev:
+                        total += m[b, h, q, v]
+                        prev = v
+                out[b, h, q] = total
+    return out

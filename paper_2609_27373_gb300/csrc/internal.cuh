@@ -75,4 +75,17 @@ int launch_attention(const wise_shape_t* sh, const void* Q, const void* K, const
 // Defined in select.cu.
 cudaError_t launch_select(const SelectParams& p, cudaStream_t stream);
 
+struct SupportMassParams {
+  long long rows;  // batch * n_heads * n_blocks
+  int n_heads, n_kv_heads, group, n_blocks, cap;
+  const float* blockmass;
+  const int32_t* idx;
+  const int32_t* counts;
+  float* retained;
+  int* status;
+};
+
+// Defined in diag.cu.
+cudaError_t launch_support_mass(const SupportMassParams& p, cudaStream_t stream);
+
 }  // namespace wise

@@ -247,6 +247,33 @@ extern "C" int wise_select_support(const wise_shape_t* shape, const wise_select_
   return launch_select(p, stream) == cudaSuccess ? WISE_OK : WISE_ERR_CUDA;
 }
 
+extern "C" int wise_support_mass(const wise_shape_t* shape, const float* blockmass, const int32_t* idx,
+                                 const int32_t* counts, int cap, float* retained, cudaStream_t stream) {
+  int rc = check_shape(shape, false);
+  if (rc != WISE_OK) return rc;
+  if (cap <= 0) return WISE_ERR_INVALID_ARG;
+  if (shape->batch == 0 || shape->seqlen == 0) return WISE_OK;
+  if (!blockmass || !idx || !counts || !retained || !aligned(blockmass, 4) || !aligned(idx, 4) ||
+      !aligned(counts, 4) || !aligned(retained, 4))
+    return WISE_ERR_INVALID_ARG;
+  int err = WISE_OK;
+  DeviceState* ds = device_state(&err);
+  if (!ds) return err;
+  SupportMassParams p;
+  p.n_heads = shape->n_heads;
+  p.n_kv_heads = shape->n_kv_heads;
+  p.group = shape->n_heads / shape->n_kv_heads;
+  p.n_blocks = shape->seqlen / shape->block;
+  p.rows = (long long)shape->batch * shape->n_heads * p.n_blocks;
+  p.cap = cap;
+  p.blockmass = blockmass;
+  p.idx = idx;
+  p.counts = counts;
+  p.retained = retained;
+  p.status = ds->status;
+  return launch_support_mass(p, stream) == cudaSuccess ? WISE_OK : WISE_ERR_CUDA;
+}
+
 extern "C" int wise_get_status(cudaStream_t stream) {
   int err = WISE_OK;
   DeviceState* ds = device_state(&err);

@@ -27,7 +27,7 @@ WISE_SEL_TOPK = 0
 WISE_SEL_COVERAGE = 1
 
 EXPORTS = ("wise_full_attn_accumulate", "wise_full_attn_accumulate_noalloc", "wise_select_support",
-           "wise_sparse_attn", "wise_get_status", "wise_status_string", "wise_version")
+           "wise_sparse_attn", "wise_support_mass", "wise_get_status", "wise_status_string", "wise_version")
 NOALLOC_SCRATCH_BYTES = 8 << 20
 
 
@@ -101,6 +101,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
                                                           P]
         lib.wise_select_support.argtypes = [ctypes.POINTER(wise_shape_t), ctypes.POINTER(wise_select_t), P, P, P, P]
         lib.wise_sparse_attn.argtypes = [ctypes.POINTER(wise_shape_t), P, P, P, P, P, ctypes.c_int, P, P]
+        lib.wise_support_mass.argtypes = [ctypes.POINTER(wise_shape_t), P, P, P, ctypes.c_int, P, P]
         lib.wise_get_status.argtypes = [P]
         lib.wise_status_string.argtypes = [ctypes.c_int]
         lib.wise_status_string.restype = ctypes.c_char_p
@@ -204,6 +205,26 @@ def wise_sparse_attn(shape: Shape, Q, K, V, idx, counts, O, stream=None) -> None
                                  _ptr(O), _stream(stream))
     if rc != WISE_OK:
         raise WiseError(rc, "wise_sparse_attn")
+
+
+def wise_support_mass(shape: Shape, blockmass, idx, counts, retained, stream=None) -> None:
+    """Routing diagnostic: retained[b, h, q] = sum of blockmass[b, h, q, kb]
+    over the support list of the kv-group of h (fp32 [batch, n_heads, nQB]).
+    With one step's mass this is the fraction of that step's full attention
+    kept by the support."""
+    nb = shape.n_blocks
+    _check(blockmass, "blockmass", (shape.batch, shape.n_heads, nb, nb), torch.float32)
+    if idx is None or idx.dim() != 4:
+        raise ValueError("idx must be int32 [batch, n_kv_heads, nQB, cap]")
+    cap = int(idx.shape[3])
+    _check(idx, "idx", (shape.batch, shape.n_kv_heads, nb, cap), torch.int32)
+    _check(counts, "counts", (shape.batch, shape.n_kv_heads, nb), torch.int32)
+    _check(retained, "retained", (shape.batch, shape.n_heads, nb), torch.float32)
+    sh = shape.c()
+    rc = load().wise_support_mass(ctypes.byref(sh), _ptr(blockmass), _ptr(idx), _ptr(counts), cap, _ptr(retained),
+                                  _stream(stream))
+    if rc != WISE_OK:
+        raise WiseError(rc, "wise_support_mass")
 
 
 def wise_get_status(stream=None) -> int:

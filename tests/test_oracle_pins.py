@@ -342,3 +342,55 @@ def test_planted_blocks_are_recovered_on_the_tiny_workload():
                 hit += p in chosen
     assert tot > 0 and hit / tot >= 0.9
     np.testing.assert_allclose(acc.sum(-1), wl.n_discovery, atol=1e-12)
+
+
+# ---------------------------------------------------------------- retained mass (routing diagnostic)
+
+def test_retained_mass_of_the_full_support_is_one():
+    # Every admissible block kept: the retained fraction is the whole row of
+    # Eq. 5, which sums to 1 (rows of A sum to 1).
+    B, H, Hkv, L, D, blk = 1, 4, 2, 64, 16, 8
+    Q, K, V = synth.random_qkv(B, H, Hkv, L, D, seed=21)
+    _, mass = orc.full_attention(Q, K, V, blk, with_mass=True)
+    idx, counts = synth.all_blocks_support(B, Hkv, L // blk)
+    r = orc.support_mass(mass, idx, counts, H)
+    assert np.allclose(r, 1.0, atol=1e-12)
+
+
+def test_retained_mass_of_complementary_supports_adds_to_one():
+    # Split the admissible blocks of every row into two disjoint supports: the
+    # two retained fractions add to the whole row (pins that no term is lost
+    # or counted twice, and that each query head reads its own row).
+    B, H, Hkv, L, D, blk = 2, 6, 3, 96, 16, 16
+    Q, K, V = synth.random_qkv(B, H, Hkv, L, D, seed=22)
+    _, mass = orc.full_attention(Q, K, V, blk, with_mass=True)
+    nb = L // blk
+    rng = np.random.default_rng(5)
+    a = np.full((B, Hkv, nb, nb), -1, dtype=np.int32)
+    c = np.full_like(a, -1)
+    na = np.zeros((B, Hkv, nb), dtype=np.int32)
+    nc = np.zeros_like(na)
+    for b, g, q in itertools.product(range(B), range(Hkv), range(nb)):
+        pick = rng.random(q + 1) < 0.5
+        sa, sc = np.flatnonzero(pick), np.flatnonzero(~pick)
+        a[b, g, q, : len(sa)], na[b, g, q] = sa, len(sa)
+        c[b, g, q, : len(sc)], nc[b, g, q] = sc, len(sc)
+    ra = orc.support_mass(mass, a, na, H)
+    rc = orc.support_mass(mass, c, nc, H)
+    assert np.allclose(ra + rc, 1.0, atol=1e-12)
+    assert ra.min() >= 0.0 and rc.min() >= 0.0
+
+
+def test_retained_mass_hand_case_with_group_lists_and_invalid_entries():
+    # 2 query heads sharing one kv-group list; 3 query blocks.  Masses are
+    # chosen by hand; invalid entries (negative, beyond the query block, not
+    # ascending) are skipped, as the attention kernels skip them.
+    mass = np.zeros((1, 2, 3, 3))
+    mass[0, 0] = [[1.0, 0, 0], [0.25, 0.75, 0], [0.5, 0.125, 0.375]]
+    mass[0, 1] = [[1.0, 0, 0], [0.5, 0.5, 0], [0.0625, 0.4375, 0.5]]
+    idx = np.array([[[[0, -1, -1], [1, 0, 1], [-3, 2, 0]]]], dtype=np.int32)
+    counts = np.array([[[1, 3, 3]]], dtype=np.int32)
+    r = orc.support_mass(mass, idx, counts, 2)
+    # q=0: {0}; q=1: {1} (0 and the repeated 1 are not ascending); q=2: {2} (-3 and 0 after 2 skipped)
+    want = np.array([[[1.0, 0.75, 0.375], [1.0, 0.5, 0.5]]])
+    assert np.array_equal(r, want)
