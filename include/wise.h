@@ -51,6 +51,12 @@ extern "C" {
 #define WISE_SEL_TOPK 0
 #define WISE_SEL_COVERAGE 1
 
+/* Modes of wise_select_working_set. */
+#define WISE_WS_UNION 0
+#define WISE_WS_STATIC 1
+#define WISE_WS_MASS_MATCHED 2
+#define WISE_WS_SIZE_MATCHED 3
+
 /* Problem geometry (Sec. 3: n = seqlen, d_h = head_dim; Sec. 5.1: block B). */
 typedef struct {
   int batch;
@@ -140,6 +146,35 @@ int wise_full_attn_accumulate_noalloc(const wise_shape_t* shape, const void* Q, 
  * counts: int32 [batch, n_kv_heads, nQB]. */
 int wise_select_support(const wise_shape_t* shape, const wise_select_t* sel, const float* blockmass,
                         int32_t* idx, int32_t* counts, cudaStream_t stream);
+
+/* Working sets of the paper's own form and its intervention controls
+ * (Eq. 6 with the union over the discovery window; appendix "Experimental
+ * details", intervention controls).  Per (batch, kv head, query block q),
+ * on the masses of the group's query heads pooled in the fixed point of
+ * wise_select_support, with admissible blocks 0..q ranked by pooled mass
+ * (descending, then block index ascending), forced blocks
+ * F = {0..n_sink-1} U {q-n_local+1..q} in every set, and a coverage set
+ * C_t(eta) = F plus candidates in rank order until the kept mass reaches eta
+ * of the admissible mass of step t:
+ *   WISE_WS_UNION         union of C_t(eta) over the n_steps given steps
+ *                         (the paper: steps t_d-3..t_d, eta = 0.95, F empty)
+ *   WISE_WS_STATIC        C_0(eta) of the one step given (Static-95)
+ *   WISE_WS_MASS_MATCHED  F plus candidates of the one step given until the
+ *                         kept mass reaches that step's mass inside the
+ *                         reference set (MassMatched)
+ *   WISE_WS_SIZE_MATCHED  F plus the top candidates of the one step given up
+ *                         to the reference set's size (SizeMatched)
+ * step_masses: fp32 [n_steps][batch][n_heads][nQB][nKB], each step's own
+ * block mass (Eq. 5, wise_full_attn_accumulate with step 0).  n_steps must
+ * be 1 except for WISE_WS_UNION.  ref_idx / ref_counts (row width ref_cap):
+ * the reference working set for the matched controls (ignored otherwise;
+ * invalid entries are skipped and reported as WISE_ERR_BAD_SUPPORT by
+ * wise_get_status).  idx / counts as wise_select_support's, with row width
+ * cap >= nKB (these sets have no size bound).  n_sink, n_local >= 0. */
+int wise_select_working_set(const wise_shape_t* shape, int mode, float eta, int n_sink, int n_local,
+                            const float* step_masses, int n_steps, const int32_t* ref_idx,
+                            const int32_t* ref_counts, int ref_cap, int32_t* idx, int32_t* counts, int cap,
+                            cudaStream_t stream);
 
 /* Routing diagnostic (appendix "Experimental details", evaluation metrics:
  * retained future attention mass).  For every query-head row (b, h, q):

@@ -186,3 +186,93 @@ def support_mass(blockmass, idx, counts, n_heads):
                         prev = v
                 out[b, h, q] = total
     return out
+
+
+def _mass_units(x):
+    """Fixed-point mass of the selection rule: floor(min(x, 4096) * 2^32) for
+    x > 0, else 0 (exact for fp32 inputs)."""
+    x = float(np.float32(x))
+    if not x > 0.0:
+        return 0
+    return int(np.floor(min(x, 4096.0) * 4294967296.0))
+
+
+def working_set(mode, step_masses, n_kv_heads, eta=0.95, n_sink=0, n_local=0, ref_idx=None, ref_counts=None):
+    """Working sets of Eq. 6 (the union over the discovery window of each
+    step's smallest block set reaching eta of the mass) and the intervention
+    controls of the appendix ("Experimental details"): Static (the first
+    step's eta set), MassMatched (the first step's smallest top set whose mass
+    reaches the first-step mass of a reference working set) and SizeMatched
+    (the first step's top blocks, as many as the reference set holds).
+
+    Same arithmetic as the selection rule of select_support: masses pooled
+    over the kv-group's query heads in exact fixed point, ranking by pooled
+    mass (descending) then block (ascending), forced blocks
+    {0..n_sink-1} U {q-n_local+1..q} in every set, coverage reached when
+    cum * 65536 >= floor(eta * 65536 + 0.5) * admissible total.
+
+    step_masses [n_steps,B,H,nQB,nKB] fp32 (mode 0 may use several steps,
+    the others exactly one).  Returns idx [B,Hkv,nQB,nQB] int32 (ascending,
+    -1 padded) and counts [B,Hkv,nQB].
+    """
+    m = np.asarray(step_masses, dtype=np.float32)
+    S, B, H, nq, nk = m.shape
+    if nq != nk or H % n_kv_heads:
+        raise ValueError("bad shapes")
+    if mode != 0 and S != 1:
+        raise ValueError("one step for the controls")
+    group = H // n_kv_heads
+    eta16 = int(np.floor(float(np.float32(eta)) * 65536.0 + 0.5))
+    idx = np.full((B, n_kv_heads, nq, nq), -1, dtype=np.int32)
+    counts = np.zeros((B, n_kv_heads, nq), dtype=np.int32)
+    for b in range(B):
+        for g in range(n_kv_heads):
+            for q in range(nq):
+                adm = list(range(q + 1))
+                forced = {kb for kb in adm if kb < n_sink or kb > q - n_local}
+
+                def pooled(st):
+                    return {kb: sum(_mass_units(m[st, b, h, q, kb]) for h in range(g * group, (g + 1) * group))
+                            for kb in adm}
+
+                def ranked(U):
+                    return sorted((kb for kb in adm if kb not in forced), key=lambda kb: (-U[kb], kb))
+
+                if mode in (0, 1):
+                    chosen = set(forced)
+                    for st in range(S):
+                        U = pooled(st)
+                        total = sum(U.values())
+                        cum = sum(U[kb] for kb in forced)
+                        sel = set(forced)
+                        for kb in ranked(U):
+                            if cum * 65536 >= eta16 * total:
+                                break
+                            sel.add(kb)
+                            cum += U[kb]
+                        chosen |= sel
+                else:
+                    U = pooled(0)
+                    n = min(max(int(ref_counts[b, g, q]), 0), ref_idx.shape[3])
+                    ref, prev = [], -1
+                    for v in ref_idx[b, g, q, :n]:
+                        v = int(v)
+                        if 0 <= v <= q and v > prev:
+                            ref.append(v)
+                            prev = v
+                    chosen = set(forced)
+                    cum = sum(U[kb] for kb in forced)
+                    if mode == 2:
+                        target = sum(U[kb] for kb in ref)
+                        for kb in ranked(U):
+                            if cum >= target:
+                                break
+                            chosen.add(kb)
+                            cum += U[kb]
+                    else:
+                        for kb in ranked(U)[: max(0, len(ref) - len(forced))]:
+                            chosen.add(kb)
+                s = sorted(chosen)
+                idx[b, g, q, : len(s)] = s
+                counts[b, g, q] = len(s)
+    return idx, counts

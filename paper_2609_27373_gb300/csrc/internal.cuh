@@ -75,6 +75,23 @@ int launch_attention(const wise_shape_t* sh, const void* Q, const void* K, const
 // Defined in select.cu.
 cudaError_t launch_select(const SelectParams& p, cudaStream_t stream);
 
+// Working-set construction of the paper's own form and its controls
+// (wise_select_working_set).
+struct WorkingSetParams {
+  int batch, n_heads, n_kv_heads, group, n_blocks;
+  int n_sink, n_local, mode, n_steps, cap, ref_cap;
+  uint64_t eta16;           // floor(eta * 65536 + 0.5)
+  const float* masses;      // [n_steps][batch][n_heads][nQB][nKB]
+  const int32_t* ref_idx;   // reference working set (mass / size matched)
+  const int32_t* ref_counts;
+  int32_t* idx;
+  int32_t* counts;
+  int* status;
+};
+
+// Defined in select.cu.
+cudaError_t launch_working_set(const WorkingSetParams& p, cudaStream_t stream);
+
 struct SupportMassParams {
   long long rows;  // batch * n_heads * n_blocks
   int n_heads, n_kv_heads, group, n_blocks, cap;

@@ -247,6 +247,50 @@ extern "C" int wise_select_support(const wise_shape_t* shape, const wise_select_
   return launch_select(p, stream) == cudaSuccess ? WISE_OK : WISE_ERR_CUDA;
 }
 
+extern "C" int wise_select_working_set(const wise_shape_t* shape, int mode, float eta, int n_sink, int n_local,
+                                       const float* step_masses, int n_steps, const int32_t* ref_idx,
+                                       const int32_t* ref_counts, int ref_cap, int32_t* idx, int32_t* counts,
+                                       int cap, cudaStream_t stream) {
+  int rc = check_shape(shape, false);
+  if (rc != WISE_OK) return rc;
+  if (mode < WISE_WS_UNION || mode > WISE_WS_SIZE_MATCHED) return WISE_ERR_INVALID_ARG;
+  if (n_sink < 0 || n_local < 0) return WISE_ERR_INVALID_ARG;
+  if (mode <= WISE_WS_STATIC && !(eta >= 0.0f && eta <= 1.0f)) return WISE_ERR_INVALID_ARG;
+  if (mode == WISE_WS_UNION ? n_steps < 1 : n_steps != 1) return WISE_ERR_INVALID_ARG;
+  const int n_blocks = shape->seqlen / shape->block;
+  if (shape->batch == 0 || shape->seqlen == 0) return WISE_OK;
+  if (n_blocks > 1024) return WISE_ERR_UNSUPPORTED;
+  if (cap < n_blocks) return WISE_ERR_INVALID_ARG;
+  if (!step_masses || !idx || !counts || !aligned(step_masses, 4) || !aligned(idx, 4) || !aligned(counts, 4))
+    return WISE_ERR_INVALID_ARG;
+  if (mode >= WISE_WS_MASS_MATCHED &&
+      (!ref_idx || !ref_counts || ref_cap <= 0 || !aligned(ref_idx, 4) || !aligned(ref_counts, 4)))
+    return WISE_ERR_INVALID_ARG;
+  int err = WISE_OK;
+  DeviceState* ds = device_state(&err);
+  if (!ds) return err;
+  WorkingSetParams p;
+  p.batch = shape->batch;
+  p.n_heads = shape->n_heads;
+  p.n_kv_heads = shape->n_kv_heads;
+  p.group = shape->n_heads / shape->n_kv_heads;
+  p.n_blocks = n_blocks;
+  p.n_sink = n_sink;
+  p.n_local = n_local;
+  p.mode = mode;
+  p.n_steps = n_steps;
+  p.cap = cap;
+  p.ref_cap = mode >= WISE_WS_MASS_MATCHED ? ref_cap : 1;
+  p.eta16 = (uint64_t)floor((double)eta * 65536.0 + 0.5);
+  p.masses = step_masses;
+  p.ref_idx = ref_idx;
+  p.ref_counts = ref_counts;
+  p.idx = idx;
+  p.counts = counts;
+  p.status = ds->status;
+  return launch_working_set(p, stream) == cudaSuccess ? WISE_OK : WISE_ERR_CUDA;
+}
+
 extern "C" int wise_support_mass(const wise_shape_t* shape, const float* blockmass, const int32_t* idx,
                                  const int32_t* counts, int cap, float* retained, cudaStream_t stream) {
   int rc = check_shape(shape, false);

@@ -27,7 +27,8 @@ WISE_SEL_TOPK = 0
 WISE_SEL_COVERAGE = 1
 
 EXPORTS = ("wise_full_attn_accumulate", "wise_full_attn_accumulate_noalloc", "wise_select_support",
-           "wise_sparse_attn", "wise_support_mass", "wise_get_status", "wise_status_string", "wise_version")
+           "wise_sparse_attn", "wise_support_mass", "wise_select_working_set", "wise_get_status",
+           "wise_status_string", "wise_version")
 NOALLOC_SCRATCH_BYTES = 8 << 20
 
 
@@ -102,6 +103,9 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.wise_select_support.argtypes = [ctypes.POINTER(wise_shape_t), ctypes.POINTER(wise_select_t), P, P, P, P]
         lib.wise_sparse_attn.argtypes = [ctypes.POINTER(wise_shape_t), P, P, P, P, P, ctypes.c_int, P, P]
         lib.wise_support_mass.argtypes = [ctypes.POINTER(wise_shape_t), P, P, P, ctypes.c_int, P, P]
+        I = ctypes.c_int
+        lib.wise_select_working_set.argtypes = [ctypes.POINTER(wise_shape_t), I, ctypes.c_float, I, I, P, I, P, P,
+                                                I, P, P, I, P]
         lib.wise_get_status.argtypes = [P]
         lib.wise_status_string.argtypes = [ctypes.c_int]
         lib.wise_status_string.restype = ctypes.c_char_p
@@ -225,6 +229,39 @@ def wise_support_mass(shape: Shape, blockmass, idx, counts, retained, stream=Non
                                   _stream(stream))
     if rc != WISE_OK:
         raise WiseError(rc, "wise_support_mass")
+
+
+WS_UNION, WS_STATIC, WS_MASS_MATCHED, WS_SIZE_MATCHED = 0, 1, 2, 3
+
+
+def wise_select_working_set(shape: Shape, mode: int, step_masses, idx, counts, eta: float = 0.95, n_sink: int = 0,
+                            n_local: int = 0, ref_idx=None, ref_counts=None, stream=None) -> None:
+    """The paper's working set (WS_UNION: union of the per-step eta coverage
+    sets of the given steps, Eq. 6) or one of its controls (WS_STATIC,
+    WS_MASS_MATCHED, WS_SIZE_MATCHED against ref_idx / ref_counts).
+    step_masses fp32 [n_steps, batch, n_heads, nQB, nKB]; idx int32
+    [batch, n_kv_heads, nQB, cap >= nQB], counts int32 [batch, n_kv_heads, nQB]."""
+    nb = shape.n_blocks
+    if step_masses is None or step_masses.dim() != 5:
+        raise ValueError("step_masses must be fp32 [n_steps, batch, n_heads, nQB, nKB]")
+    n_steps = int(step_masses.shape[0])
+    _check(step_masses, "step_masses", (n_steps, shape.batch, shape.n_heads, nb, nb), torch.float32)
+    if idx is None or idx.dim() != 4:
+        raise ValueError("idx must be int32 [batch, n_kv_heads, nQB, cap]")
+    cap = int(idx.shape[3])
+    _check(idx, "idx", (shape.batch, shape.n_kv_heads, nb, cap), torch.int32)
+    _check(counts, "counts", (shape.batch, shape.n_kv_heads, nb), torch.int32)
+    ref_cap = 0
+    if ref_idx is not None:
+        ref_cap = int(ref_idx.shape[3])
+        _check(ref_idx, "ref_idx", (shape.batch, shape.n_kv_heads, nb, ref_cap), torch.int32)
+        _check(ref_counts, "ref_counts", (shape.batch, shape.n_kv_heads, nb), torch.int32)
+    sh = shape.c()
+    rc = load().wise_select_working_set(ctypes.byref(sh), int(mode), float(eta), int(n_sink), int(n_local),
+                                        _ptr(step_masses), n_steps, _ptr(ref_idx), _ptr(ref_counts), ref_cap,
+                                        _ptr(idx), _ptr(counts), cap, _stream(stream))
+    if rc != WISE_OK:
+        raise WiseError(rc, "wise_select_working_set")
 
 
 def wise_get_status(stream=None) -> int:

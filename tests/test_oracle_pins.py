@@ -394,3 +394,113 @@ def test_retained_mass_hand_case_with_group_lists_and_invalid_entries():
     # q=0: {0}; q=1: {1} (0 and the repeated 1 are not ascending); q=2: {2} (-3 and 0 after 2 skipped)
     want = np.array([[[1.0, 0.75, 0.375], [1.0, 0.5, 0.5]]])
     assert np.array_equal(r, want)
+
+
+# ---------------------------------------------------------------- working sets of Eq. 6 and the controls
+
+def _ws_units(x):
+    x = float(np.float32(x))
+    return 0 if not x > 0 else int(math.floor(min(x, 4096.0) * 2.0 ** 32))
+
+
+def _rows(masses, group):
+    """Pooled fixed-point masses per (step, b, g, q) row, for brute force."""
+    S, B, H, nq, _ = masses.shape
+    for st, b, g, q in itertools.product(range(S), range(B), range(H // group), range(nq)):
+        yield st, b, g, q, [sum(_ws_units(masses[st, b, h, q, kb]) for h in range(g * group, (g + 1) * group))
+                            for kb in range(q + 1)]
+
+
+def _min_cover(U, forced, need):
+    """Exhaustive search: the smallest size of a set holding `forced` whose
+    mass satisfies need(mass)."""
+    rest = [kb for kb in range(len(U)) if kb not in forced]
+    for k in range(len(rest) + 1):
+        for extra in itertools.combinations(rest, k):
+            if need(sum(U[kb] for kb in forced) + sum(U[kb] for kb in extra)):
+                return len(forced) + k
+    return None
+
+
+@pytest.mark.parametrize("n_sink,n_local", [(0, 0), (1, 1)])
+def test_static_set_is_a_minimum_eta_cover_by_exhaustive_search(n_sink, n_local):
+    rng = np.random.default_rng(31)
+    masses = rng.dirichlet(np.ones(7), size=(1, 1, 2, 7)).astype(np.float32)  # rows of 7 blocks
+    masses = np.tril(masses.reshape(1, 1, 2, 7, 7))  # only admissible blocks kb <= q carry mass
+    eta = 0.8
+    eta16 = int(math.floor(float(np.float32(eta)) * 65536 + 0.5))
+    idx, counts = orc.working_set(1, masses, 2, eta=eta, n_sink=n_sink, n_local=n_local)
+    for _, b, g, q, U in _rows(masses, 1):
+        forced = {kb for kb in range(q + 1) if kb < n_sink or kb > q - n_local}
+        total = sum(U)
+        sel = idx[b, g, q, : counts[b, g, q]]
+        assert set(forced) <= set(sel.tolist())
+        assert sum(U[kb] for kb in sel) * 65536 >= eta16 * total
+        assert counts[b, g, q] == _min_cover(U, forced, lambda s: s * 65536 >= eta16 * total)
+
+
+def test_union_is_the_union_of_the_per_step_sets():
+    rng = np.random.default_rng(32)
+    masses = np.tril(rng.random((3, 1, 2, 6, 6))).astype(np.float32)
+    masses /= masses.sum(-1, keepdims=True)
+    u_idx, u_cnt = orc.working_set(0, masses, 1, eta=0.9, n_sink=1, n_local=1)
+    per = [orc.working_set(1, masses[s:s + 1], 1, eta=0.9, n_sink=1, n_local=1) for s in range(3)]
+    for b, g, q in itertools.product(range(1), range(1), range(6)):
+        want = set()
+        for idx, cnt in per:
+            want |= set(idx[b, g, q, : cnt[b, g, q]].tolist())
+        assert sorted(want) == u_idx[b, g, q, : u_cnt[b, g, q]].tolist()
+    # the same step twice adds nothing
+    twice = np.concatenate([masses[:1], masses[:1]])
+    a = orc.working_set(0, twice, 1, eta=0.9)
+    b1 = orc.working_set(1, masses[:1], 1, eta=0.9)
+    assert np.array_equal(a[0], b1[0]) and np.array_equal(a[1], b1[1])
+
+
+def test_mass_and_size_matched_controls_by_exhaustive_search():
+    rng = np.random.default_rng(33)
+    nq = 7
+    masses = np.tril(rng.random((1, 1, 3, nq, nq))).astype(np.float32)
+    masses /= masses.sum(-1, keepdims=True)
+    # reference working set: a random admissible subset of each row
+    ref_idx = np.full((1, 3, nq, nq), -1, dtype=np.int32)
+    ref_cnt = np.zeros((1, 3, nq), dtype=np.int32)
+    for g, q in itertools.product(range(3), range(nq)):
+        s = sorted(rng.choice(q + 1, size=rng.integers(1, q + 2), replace=False).tolist())
+        ref_idx[0, g, q, : len(s)], ref_cnt[0, g, q] = s, len(s)
+    mm = orc.working_set(2, masses, 3, ref_idx=ref_idx, ref_counts=ref_cnt)
+    sm = orc.working_set(3, masses, 3, ref_idx=ref_idx, ref_counts=ref_cnt)
+    for _, b, g, q, U in _rows(masses, 1):
+        ref = ref_idx[b, g, q, : ref_cnt[b, g, q]].tolist()
+        target = sum(U[kb] for kb in ref)
+        m_sel = mm[0][b, g, q, : mm[1][b, g, q]].tolist()
+        assert sum(U[kb] for kb in m_sel) >= target
+        assert len(m_sel) == _min_cover(U, set(), lambda s: s >= target) <= len(ref)
+        s_sel = sm[0][b, g, q, : sm[1][b, g, q]].tolist()
+        assert len(s_sel) == len(ref)
+        best = max(sum(U[kb] for kb in c) for c in itertools.combinations(range(q + 1), len(ref)))
+        assert sum(U[kb] for kb in s_sel) == best
+    # against its own coverage set, the mass-matched control is that set
+    st = orc.working_set(1, masses, 3, eta=0.9)
+    same = orc.working_set(2, masses, 3, ref_idx=st[0], ref_counts=st[1])
+    assert np.array_equal(same[0], st[0]) and np.array_equal(same[1], st[1])
+
+
+def test_working_set_hand_case_with_gqa_pooling():
+    # 2 query heads pooled into one kv group, one step, q = 3 (4 admissible
+    # blocks).  Pooled masses (halves): head 0 [0.5, 0.25, 0.125, 0.125],
+    # head 1 [0.125, 0.5, 0.25, 0.125] -> pooled [0.625, 0.75, 0.375, 0.25] of
+    # total 2.  eta = 0.6 needs 1.2: ranked 1 (0.75), 0 (0.625) -> {0, 1}.
+    m = np.zeros((1, 1, 2, 4, 4), dtype=np.float32)
+    m[0, 0, 0, 3] = [0.5, 0.25, 0.125, 0.125]
+    m[0, 0, 1, 3] = [0.125, 0.5, 0.25, 0.125]
+    idx, counts = orc.working_set(1, m, 1, eta=0.6)
+    assert idx[0, 0, 3, : counts[0, 0, 3]].tolist() == [0, 1]
+    # with the diagonal forced: {3} holds 0.25, then 1 (1.0), then 0 (1.625 >= 1.2)
+    idx, counts = orc.working_set(1, m, 1, eta=0.6, n_local=1)
+    assert idx[0, 0, 3, : counts[0, 0, 3]].tolist() == [0, 1, 3]
+    # size matched against a 2-block reference with the diagonal forced: {3} + top 1 -> {1, 3}
+    ref = np.array([[[[0, 2, -1, -1]] * 4]], dtype=np.int32)
+    rc = np.full((1, 1, 4), 2, dtype=np.int32)
+    idx, counts = orc.working_set(3, m, 1, n_local=1, ref_idx=ref, ref_counts=rc)
+    assert idx[0, 0, 3, : counts[0, 0, 3]].tolist() == [1, 3]
