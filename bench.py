@@ -390,6 +390,41 @@ def main():
         ret.append(float(retained.mean()))
     retained_mass = statistics.mean(ret)
 
+    # ---- the paper's own working set (union over the discovery window of each
+    # step's 95 % coverage set, Eq. 6) and the intervention controls, each with
+    # its density, retained late-step mass and late-step sparse time
+    step_mass = torch.empty((wl.n_discovery, wl.batch, wl.n_heads, nb, nb), dtype=torch.float32, device="cuda")
+    for t in range(wl.n_discovery):
+        wise.wise_full_attn_accumulate(shape, *dev_steps[t], O, step_mass[t], 0)
+    ws_idx = {k: torch.empty((wl.batch, wl.n_kv_heads, nb, nb), dtype=torch.int32, device="cuda")
+              for k in ("union", "static", "mass_matched", "size_matched")}
+    ws_cnt = {k: torch.empty((wl.batch, wl.n_kv_heads, nb), dtype=torch.int32, device="cuda") for k in ws_idx}
+    forced = dict(n_sink=wl.n_sink, n_local=wl.n_local)
+    wise.wise_select_working_set(shape, wise.WS_UNION, step_mass, ws_idx["union"], ws_cnt["union"], eta=wl.eta,
+                                 **forced)
+    wise.wise_select_working_set(shape, wise.WS_STATIC, step_mass[:1], ws_idx["static"], ws_cnt["static"],
+                                 eta=wl.eta, **forced)
+    for k, mode in (("mass_matched", wise.WS_MASS_MATCHED), ("size_matched", wise.WS_SIZE_MATCHED)):
+        wise.wise_select_working_set(shape, mode, step_mass[:1], ws_idx[k], ws_cnt[k], ref_idx=ws_idx["union"],
+                                     ref_counts=ws_cnt["union"], **forced)
+    admissible = wl.batch * wl.n_kv_heads * nb * (nb + 1) / 2
+    supports = {}
+    for k in ws_idx:
+        rm = []
+        for t in range(wl.n_discovery, wl.steps, 4):
+            wise.wise_full_attn_accumulate(shape, *dev_steps[t], O, diag_mass, 0)
+            wise.wise_support_mass(shape, diag_mass, ws_idx[k], ws_cnt[k], retained)
+            rm.append(float(retained.mean()))
+        evs_k = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_late)]
+        for i, t in enumerate(range(wl.n_discovery, wl.steps)):
+            evs_k[i][0].record(stream)
+            wise.wise_sparse_attn(shape, *dev_steps[t], ws_idx[k], ws_cnt[k], O)
+            evs_k[i][1].record(stream)
+        torch.cuda.synchronize()
+        supports[k] = {"density": round(float(ws_cnt[k].sum()) / admissible, 4),
+                       "retained_mass": round(statistics.mean(rm), 4),
+                       "sparse_ms": round(statistics.mean(a.elapsed_time(b) for a, b in evs_k), 5)}
+
     # ---- the whole trajectory as one CUDA graph (discovery, selection, late
     # steps), replayed; its launches carry no host-side gaps
     graph = {"ms": None, "note": None}
@@ -457,6 +492,8 @@ def main():
         "density": round(density, 4),
         "retained_mass": round(retained_mass, 4),
         "all_blocks_ms": round(all_blocks_ms, 5),
+        "block_density": round(float(layer.counts.sum()) / (wl.batch * wl.n_kv_heads * nb * (nb + 1) / 2), 4),
+        "supports": supports,
         "all_blocks_vs_dense": round(all_blocks_ms / dense, 4),
         "graph_trajectory_ms": None if graph["ms"] is None else round(graph["ms"], 4),
         "graph_trajectory_speedup": None if graph["ms"] is None else round(wl.steps * dense / graph["ms"], 4),
