@@ -425,6 +425,31 @@ def main():
                        "retained_mass": round(statistics.mean(rm), 4),
                        "sparse_ms": round(statistics.mean(a.elapsed_time(b) for a, b in evs_k), 5)}
 
+    # ---- stability of the rolling working set at the discovery endpoint
+    # (appendix "Stability of the Deployed Working Set"): W(t) = union of the
+    # eta sets of steps t-3..t; Jaccard of W(t_d - 1) and W(t_d)
+    roll = []
+    for t in (wl.n_discovery - 2, wl.n_discovery - 1):
+        r_idx = torch.empty((wl.batch, wl.n_kv_heads, nb, nb), dtype=torch.int32, device="cuda")
+        r_cnt = torch.empty((wl.batch, wl.n_kv_heads, nb), dtype=torch.int32, device="cuda")
+        wise.wise_select_working_set(shape, wise.WS_UNION, step_mass[max(0, t - 3):t + 1].contiguous(), r_idx, r_cnt,
+                                     eta=wl.eta, **forced)
+        roll.append((r_idx, r_cnt))
+    inter_union = torch.empty((wl.batch, 2), dtype=torch.int64, device="cuda")
+    wise.wise_support_overlap(shape, roll[0][0], roll[0][1], roll[1][0], roll[1][1], inter_union)
+    rolling_jaccard = statistics.mean(1.0 if u == 0 else i / u for i, u in inter_union.cpu().tolist())
+
+    # ---- Freeze-A control: the selected support with the within-support
+    # distribution of the last discovery step, applied to each late step's V
+    fz_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_late)]
+    Q_td, K_td, _ = dev_steps[wl.n_discovery - 1]
+    for i, t in enumerate(range(wl.n_discovery, wl.steps)):
+        fz_ev[i][0].record(stream)
+        wise.wise_freeze_a_attn(shape, Q_td, K_td, dev_steps[t][2], layer.idx, layer.counts, O)
+        fz_ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    freeze_a_ms = statistics.mean(a.elapsed_time(b) for a, b in fz_ev)
+
     # ---- the whole trajectory as one CUDA graph (discovery, selection, late
     # steps), replayed; its launches carry no host-side gaps
     graph = {"ms": None, "note": None}
@@ -494,6 +519,8 @@ def main():
         "all_blocks_ms": round(all_blocks_ms, 5),
         "block_density": round(float(layer.counts.sum()) / (wl.batch * wl.n_kv_heads * nb * (nb + 1) / 2), 4),
         "supports": supports,
+        "rolling_jaccard_at_discovery_end": round(rolling_jaccard, 4),
+        "freeze_a_ms": round(freeze_a_ms, 5),
         "all_blocks_vs_dense": round(all_blocks_ms / dense, 4),
         "graph_trajectory_ms": None if graph["ms"] is None else round(graph["ms"], 4),
         "graph_trajectory_speedup": None if graph["ms"] is None else round(wl.steps * dense / graph["ms"], 4),

@@ -205,6 +205,38 @@ int wise_support_mass(const wise_shape_t* shape, const float* blockmass, const i
 int wise_sparse_attn(const wise_shape_t* shape, const void* Q, const void* K, const void* V, const int32_t* idx,
                      const int32_t* counts, int cap, void* O, cudaStream_t stream);
 
+/* Freeze-A control (appendix "Experimental details", intervention controls):
+ * the support W of WISE, with the within-support attention distribution frozen
+ * at a past step t0 (the discovery endpoint):
+ *   Abar_ij = A(t0)_ij [b(j) in W_q(i)] / sum_k A(t0)_ik [b(k) in W_q(i)],
+ *   O = Abar V,
+ * where A(t0) is that step's unrestricted causal attention and V the current
+ * step's values.  The full-attention normaliser cancels in Abar, so Abar is
+ * the softmax of scale * Q(t0) K(t0)^T + M + R over the support (Eqs. 7-8 with
+ * the frozen Q and K): Q_frozen and K_frozen are step t0's queries and keys,
+ * V the current values, all in the layouts of wise_sparse_attn, which this
+ * call runs; idx, counts, cap, O, errors and the treatment of malformed lists
+ * as there. */
+int wise_freeze_a_attn(const wise_shape_t* shape, const void* Q_frozen, const void* K_frozen, const void* V,
+                       const int32_t* idx, const int32_t* counts, int cap, void* O, cudaStream_t stream);
+
+/* Overlap of two block supports A and B (e.g. the rolling working sets of two
+ * consecutive steps, appendix "Stability of the Deployed Working Set"): for
+ * each batch element e, over all (kv head, query block) rows,
+ *   inter_union[2e]     = number of (row, key block) pairs in both A and B,
+ *   inter_union[2e + 1] = number in A or B,
+ * so that the element's rolling-set Jaccard is inter / union (defined as 1
+ * when both are empty).  idx_a/counts_a (row width cap_a) and idx_b/counts_b
+ * (row width cap_b): layouts of wise_select_support's output.  inter_union:
+ * device, 2 * batch unsigned 64-bit integers, 8-byte aligned, overwritten.
+ * Exact integer counts.  List entries are used as the attention kernels use
+ * them: malformed entries are skipped and flagged as WISE_ERR_BAD_SUPPORT.
+ * Errors: INVALID_ARG for NULL or misaligned pointers or a cap <= 0; the shape
+ * rules of wise_select_support (head_dim unused). */
+int wise_support_overlap(const wise_shape_t* shape, const int32_t* idx_a, const int32_t* counts_a, int cap_a,
+                         const int32_t* idx_b, const int32_t* counts_b, int cap_b, unsigned long long* inter_union,
+                         cudaStream_t stream);
+
 /* Synchronizes `stream`, then reads and clears the current device's status
  * word: WISE_OK, WISE_ERR_BAD_SUPPORT or WISE_ERR_TIMEOUT (the latter wins
  * when both were recorded), or WISE_ERR_CUDA if the synchronization failed. */

@@ -276,3 +276,73 @@ def working_set(mode, step_masses, n_kv_heads, eta=0.95, n_sink=0, n_local=0, re
                 idx[b, g, q, : len(s)] = s
                 counts[b, g, q] = len(s)
     return idx, counts
+
+
+def _used_blocks(idx_row, n, q):
+    """Entries of a support list that the attention kernels use: the first n
+    (clamped to the row width), skipping entries that are negative, beyond
+    query block q or not strictly above the last accepted entry."""
+    n = min(max(int(n), 0), len(idx_row))
+    out, prev = [], -1
+    for v in idx_row[:n]:
+        v = int(v)
+        if 0 <= v <= q and v > prev:
+            out.append(v)
+            prev = v
+    return out
+
+
+def support_overlap(idx_a, counts_a, idx_b, counts_b):
+    """Overlap of two block supports (appendix "Stability of the Deployed
+    Working Set"): the working set of an example is the collection of active
+    (head, query block, key block) triples, and the rolling-set Jaccard of two
+    consecutive steps is |W(t-1) & W(t)| / |W(t-1) | W(t)|.  Returns int64
+    [B, 2]: per batch element the sizes of the intersection and of the union,
+    from Python sets.  idx [B,Hkv,nQB,cap], counts [B,Hkv,nQB]."""
+    B, Hkv, nq = np.asarray(counts_a).shape
+    out = np.zeros((B, 2), dtype=np.int64)
+    for b in range(B):
+        wa, wb = set(), set()
+        for g in range(Hkv):
+            for q in range(nq):
+                wa.update((g, q, v) for v in _used_blocks(idx_a[b, g, q], counts_a[b, g, q], q))
+                wb.update((g, q, v) for v in _used_blocks(idx_b[b, g, q], counts_b[b, g, q], q))
+        out[b, 0] = len(wa & wb)
+        out[b, 1] = len(wa | wb)
+    return out
+
+
+def freeze_a(Q0, K0, V, idx, counts, block, scale=None):
+    """Freeze-A control (appendix "Experimental details", intervention
+    controls), in the order the paper defines it: A = the unrestricted causal
+    attention of the frozen step (softmax of scale * Q0 K0^T + M, Eq. 2),
+    Abar = A restricted to the key blocks of the support and renormalised over
+    the admissible keys, O = Abar V with the current step's V.  fp64 numpy.
+    Q0 [B,H,L,d], K0 and V [B,Hkv,L,d] (any float dtype), idx [B,Hkv,nQB,cap],
+    counts [B,Hkv,nQB].  Rows whose restricted mass is zero give O = 0."""
+    Q0 = np.asarray(Q0, dtype=np.float64)
+    K0 = np.asarray(K0, dtype=np.float64)
+    V = np.asarray(V, dtype=np.float64)
+    B, H, L, d = Q0.shape
+    Hkv = K0.shape[1]
+    group = H // Hkv
+    sc = 1.0 / np.sqrt(d) if scale is None else float(scale)
+    nq = L // block
+    causal = np.tril(np.ones((L, L), dtype=bool))
+    out = np.zeros((B, H, L, V.shape[3]), dtype=np.float64)
+    for b in range(B):
+        for h in range(H):
+            g = h // group
+            s = sc * (Q0[b, h] @ K0[b, g].T)
+            s = np.where(causal, s, -np.inf)
+            a = np.exp(s - s.max(axis=1, keepdims=True))
+            a /= a.sum(axis=1, keepdims=True)
+            keep = np.zeros((L, L), dtype=bool)
+            for q in range(nq):
+                for v in _used_blocks(idx[b, g, q], counts[b, g, q], q):
+                    keep[q * block:(q + 1) * block, v * block:(v + 1) * block] = True
+            abar = np.where(keep & causal, a, 0.0)
+            tot = abar.sum(axis=1, keepdims=True)
+            abar = np.divide(abar, tot, out=np.zeros_like(abar), where=tot > 0)
+            out[b, h] = abar @ V[b, g]
+    return out

@@ -102,7 +102,19 @@ struct SupportMassParams {
   int* status;
 };
 
+struct SupportOverlapParams {
+  int batch, rows;  // rows per batch element: n_kv_heads * n_blocks
+  int n_blocks, cap_a, cap_b;
+  const int32_t* idx_a;
+  const int32_t* counts_a;
+  const int32_t* idx_b;
+  const int32_t* counts_b;
+  unsigned long long* inter_union;  // [batch][2]
+  int* status;
+};
+
 // Defined in diag.cu.
 cudaError_t launch_support_mass(const SupportMassParams& p, cudaStream_t stream);
+cudaError_t launch_support_overlap(const SupportOverlapParams& p, cudaStream_t stream);
 
 }  // namespace wise

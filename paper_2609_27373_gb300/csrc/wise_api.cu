@@ -1,5 +1,6 @@
 // Host side of the C ABI declared in include/wise.h: argument checks, TMA
 // tensor maps, the per-device scratch buffer and status word, and launches.
+#include <limits.h>
 #include <math.h>
 #include <mutex>
 
@@ -213,6 +214,15 @@ extern "C" int wise_sparse_attn(const wise_shape_t* shape, const void* Q, const 
   return launch_attention(shape, Q, K, V, O, kSparse, nullptr, 0, idx, counts, cap, stream);
 }
 
+extern "C" int wise_freeze_a_attn(const wise_shape_t* shape, const void* Q_frozen, const void* K_frozen,
+                                  const void* V, const int32_t* idx, const int32_t* counts, int cap, void* O,
+                                  cudaStream_t stream) {
+  // The frozen distribution restricted to the support and renormalised is the
+  // softmax over the support of the frozen step's logits, so the sparse kernel
+  // computes it from that step's Q and K against the current V.
+  return launch_attention(shape, Q_frozen, K_frozen, V, O, kSparse, nullptr, 0, idx, counts, cap, stream);
+}
+
 extern "C" int wise_select_support(const wise_shape_t* shape, const wise_select_t* sel, const float* blockmass,
                                    int32_t* idx, int32_t* counts, cudaStream_t stream) {
   int rc = check_shape(shape, false);
@@ -316,6 +326,37 @@ extern "C" int wise_support_mass(const wise_shape_t* shape, const float* blockma
   p.retained = retained;
   p.status = ds->status;
   return launch_support_mass(p, stream) == cudaSuccess ? WISE_OK : WISE_ERR_CUDA;
+}
+
+extern "C" int wise_support_overlap(const wise_shape_t* shape, const int32_t* idx_a, const int32_t* counts_a,
+                                    int cap_a, const int32_t* idx_b, const int32_t* counts_b, int cap_b,
+                                    unsigned long long* inter_union, cudaStream_t stream) {
+  int rc = check_shape(shape, false);
+  if (rc != WISE_OK) return rc;
+  if (cap_a <= 0 || cap_b <= 0) return WISE_ERR_INVALID_ARG;
+  if (shape->batch == 0) return WISE_OK;
+  if (!inter_union || !aligned(inter_union, 8)) return WISE_ERR_INVALID_ARG;
+  const long long rows = (long long)shape->n_kv_heads * (shape->seqlen / shape->block);
+  if (rows > INT_MAX) return WISE_ERR_UNSUPPORTED;
+  if (rows > 0 && (!idx_a || !counts_a || !idx_b || !counts_b || !aligned(idx_a, 4) || !aligned(counts_a, 4) ||
+                   !aligned(idx_b, 4) || !aligned(counts_b, 4)))
+    return WISE_ERR_INVALID_ARG;
+  int err = WISE_OK;
+  DeviceState* ds = device_state(&err);
+  if (!ds) return err;
+  SupportOverlapParams p;
+  p.batch = shape->batch;
+  p.rows = (int)rows;
+  p.n_blocks = shape->seqlen / shape->block;
+  p.cap_a = cap_a;
+  p.cap_b = cap_b;
+  p.idx_a = idx_a;
+  p.counts_a = counts_a;
+  p.idx_b = idx_b;
+  p.counts_b = counts_b;
+  p.inter_union = inter_union;
+  p.status = ds->status;
+  return launch_support_overlap(p, stream) == cudaSuccess ? WISE_OK : WISE_ERR_CUDA;
 }
 
 extern "C" int wise_get_status(cudaStream_t stream) {

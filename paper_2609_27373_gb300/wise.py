@@ -27,8 +27,8 @@ WISE_SEL_TOPK = 0
 WISE_SEL_COVERAGE = 1
 
 EXPORTS = ("wise_full_attn_accumulate", "wise_full_attn_accumulate_noalloc", "wise_select_support",
-           "wise_sparse_attn", "wise_support_mass", "wise_select_working_set", "wise_get_status",
-           "wise_status_string", "wise_version")
+           "wise_sparse_attn", "wise_freeze_a_attn", "wise_support_mass", "wise_support_overlap",
+           "wise_select_working_set", "wise_get_status", "wise_status_string", "wise_version")
 NOALLOC_SCRATCH_BYTES = 8 << 20
 
 
@@ -102,8 +102,10 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
                                                           P]
         lib.wise_select_support.argtypes = [ctypes.POINTER(wise_shape_t), ctypes.POINTER(wise_select_t), P, P, P, P]
         lib.wise_sparse_attn.argtypes = [ctypes.POINTER(wise_shape_t), P, P, P, P, P, ctypes.c_int, P, P]
+        lib.wise_freeze_a_attn.argtypes = [ctypes.POINTER(wise_shape_t), P, P, P, P, P, ctypes.c_int, P, P]
         lib.wise_support_mass.argtypes = [ctypes.POINTER(wise_shape_t), P, P, P, ctypes.c_int, P, P]
         I = ctypes.c_int
+        lib.wise_support_overlap.argtypes = [ctypes.POINTER(wise_shape_t), P, P, I, P, P, I, P, P]
         lib.wise_select_working_set.argtypes = [ctypes.POINTER(wise_shape_t), I, ctypes.c_float, I, I, P, I, P, P,
                                                 I, P, P, I, P]
         lib.wise_get_status.argtypes = [P]
@@ -209,6 +211,43 @@ def wise_sparse_attn(shape: Shape, Q, K, V, idx, counts, O, stream=None) -> None
                                  _ptr(O), _stream(stream))
     if rc != WISE_OK:
         raise WiseError(rc, "wise_sparse_attn")
+
+
+def wise_freeze_a_attn(shape: Shape, Q_frozen, K_frozen, V, idx, counts, O, stream=None) -> None:
+    """Freeze-A control: the within-support attention distribution of a past
+    step (its Q and K) applied to the current V, O = Abar V."""
+    _qkvo(shape, Q_frozen, K_frozen, V, O)
+    nb = shape.n_blocks
+    if idx is None or idx.dim() != 4:
+        raise ValueError("idx must be int32 [batch, n_kv_heads, nQB, cap]")
+    cap = idx.shape[-1]
+    _check(idx, "idx", (shape.batch, shape.n_kv_heads, nb, cap), torch.int32)
+    _check(counts, "counts", (shape.batch, shape.n_kv_heads, nb), torch.int32)
+    sh = shape.c()
+    rc = load().wise_freeze_a_attn(ctypes.byref(sh), _ptr(Q_frozen), _ptr(K_frozen), _ptr(V), _ptr(idx),
+                                   _ptr(counts), int(cap), _ptr(O), _stream(stream))
+    if rc != WISE_OK:
+        raise WiseError(rc, "wise_freeze_a_attn")
+
+
+def wise_support_overlap(shape: Shape, idx_a, counts_a, idx_b, counts_b, inter_union, stream=None) -> None:
+    """inter_union int64 [batch, 2] (device; bit pattern of the C API's
+    unsigned counts) = per batch element the number of (kv head, query block,
+    key block) triples in both supports and in either."""
+    nb = shape.n_blocks
+    caps = []
+    for name, idx, counts in (("idx_a", idx_a, counts_a), ("idx_b", idx_b, counts_b)):
+        if idx is None or idx.dim() != 4:
+            raise ValueError(f"{name} must be int32 [batch, n_kv_heads, nQB, cap]")
+        caps.append(int(idx.shape[3]))
+        _check(idx, name, (shape.batch, shape.n_kv_heads, nb, caps[-1]), torch.int32)
+        _check(counts, "counts" + name[3:], (shape.batch, shape.n_kv_heads, nb), torch.int32)
+    _check(inter_union, "inter_union", (shape.batch, 2), torch.int64)
+    sh = shape.c()
+    rc = load().wise_support_overlap(ctypes.byref(sh), _ptr(idx_a), _ptr(counts_a), caps[0], _ptr(idx_b),
+                                     _ptr(counts_b), caps[1], _ptr(inter_union), _stream(stream))
+    if rc != WISE_OK:
+        raise WiseError(rc, "wise_support_overlap")
 
 
 def wise_support_mass(shape: Shape, blockmass, idx, counts, retained, stream=None) -> None:

@@ -504,3 +504,106 @@ def test_working_set_hand_case_with_gqa_pooling():
     rc = np.full((1, 1, 4), 2, dtype=np.int32)
     idx, counts = orc.working_set(3, m, 1, n_local=1, ref_idx=ref, ref_counts=rc)
     assert idx[0, 0, 3, : counts[0, 0, 3]].tolist() == [1, 3]
+
+
+# ---------------------------------------------- rolling-set overlap (appendix)
+
+def _lists(rows, cap):
+    """rows: {(g, q): [entries]} for B = 1 -> idx [1,Hkv,nQB,cap], counts."""
+    Hkv = 1 + max(g for g, _ in rows)
+    nq = 1 + max(q for _, q in rows)
+    idx = np.full((1, Hkv, nq, cap), -1, dtype=np.int32)
+    counts = np.zeros((1, Hkv, nq), dtype=np.int32)
+    for (g, q), ent in rows.items():
+        idx[0, g, q, :len(ent)] = ent
+        counts[0, g, q] = len(ent)
+    return idx, counts
+
+
+def test_overlap_hand_case_with_invalid_entries():
+    """Two supports over 2 kv heads x 3 query blocks, counted by hand: each
+    row shares exactly one block, and the rows hold 1, 2, 3 distinct blocks in
+    the union, so |A & B| = 6 and |A | B| = 12 (Jaccard 1/2).  A repeated
+    entry and an entry beyond its query block are skipped."""
+    a = {(0, 0): [0], (0, 1): [0, 1, 1], (0, 2): [0, 2], (1, 0): [0], (1, 1): [1], (1, 2): [0, 1, 2]}
+    b = {(0, 0): [0], (0, 1): [1], (0, 2): [1, 2], (1, 0): [0], (1, 1): [0, 1], (1, 2): [2, 5]}
+    ia, ca = _lists(a, 4)
+    ib, cb = _lists(b, 4)
+    np.testing.assert_array_equal(orc.support_overlap(ia, ca, ib, cb), [[6, 12]])
+    np.testing.assert_array_equal(orc.support_overlap(ib, cb, ia, ca), [[6, 12]])
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_overlap_identities_on_random_supports(seed):
+    """|A & A| = |A | A| = |A| = sum of counts for well-formed lists;
+    inclusion-exclusion |A & B| + |A | B| = |A| + |B|; supports without a
+    common block have an empty intersection."""
+    B, Hkv, nb = 2, 3, 9
+    ia, ca = synth.random_support(B, Hkv, nb, 5, seed=seed)
+    ib, cb = synth.random_support(B, Hkv, nb, 7, seed=seed + 10)
+    self_ov = orc.support_overlap(ia, ca, ia, ca)
+    np.testing.assert_array_equal(self_ov[:, 0], ca.sum(axis=(1, 2)))
+    np.testing.assert_array_equal(self_ov[:, 1], ca.sum(axis=(1, 2)))
+    ov = orc.support_overlap(ia, ca, ib, cb)
+    np.testing.assert_array_equal(ov[:, 0] + ov[:, 1], ca.sum(axis=(1, 2)) + cb.sum(axis=(1, 2)))
+    # Even blocks only against odd blocks only.
+    ev, cev = ia.copy(), ca.copy()
+    od, cod = ia.copy(), ca.copy()
+    for arr, cnt, parity in ((ev, cev, 0), (od, cod, 1)):
+        for bb in range(B):
+            for g in range(Hkv):
+                for q in range(nb):
+                    keep = [v for v in range(q + 1) if v % 2 == parity]
+                    arr[bb, g, q, :] = -1
+                    arr[bb, g, q, :len(keep[:5])] = keep[:5]
+                    cnt[bb, g, q] = len(keep[:5])
+    ov = orc.support_overlap(ev, cev, od, cod)
+    assert (ov[:, 0] == 0).all() and (ov[:, 1] == cev.sum(axis=(1, 2)) + cod.sum(axis=(1, 2))).all()
+
+
+# ------------------------------------------------------------ Freeze-A (appendix)
+
+def test_freeze_a_with_the_frozen_values_is_the_sparse_attention_of_that_step():
+    """With V = the frozen step's V, Abar V is that step's support-restricted
+    attention: softmax-then-restrict-and-renormalise (the control's definition)
+    equals restrict-then-softmax (Eqs. 7-8, the C oracle)."""
+    B, H, Hkv, L, D, blk = 2, 4, 2, 64, 8, 8
+    Q, K, V = synth.random_qkv(B, H, Hkv, L, D, seed=21)
+    idx, counts = synth.random_support(B, Hkv, L // blk, 4, seed=22)
+    got = orc.freeze_a(bf16_vals(Q), bf16_vals(K), bf16_vals(V), idx, counts, blk)
+    want = orc.sparse_attention(Q, K, V, idx, counts, blk)
+    np.testing.assert_allclose(got, want, rtol=0, atol=1e-12)
+
+
+def test_freeze_a_with_every_block_is_full_attention_on_the_new_values():
+    """With the all-blocks support Abar = A: O = A(Q0, K0) V, i.e. torch's
+    causal SDPA with the frozen Q and K and the new V."""
+    B, H, Hkv, L, D, blk = 1, 3, 3, 40, 5, 8
+    Q, K, V0 = synth.random_qkv(B, H, Hkv, L, D, seed=23)
+    _, _, V1 = synth.random_qkv(B, H, Hkv, L, D, seed=24)
+    idx, counts = synth.all_blocks_support(B, Hkv, L // blk)
+    got = orc.freeze_a(bf16_vals(Q), bf16_vals(K), bf16_vals(V1), idx, counts, blk)
+    ref = sdpa_reference(Q, K, V1, 1, is_causal=True)
+    np.testing.assert_allclose(got, ref, rtol=0, atol=1e-12)
+
+
+def test_freeze_a_rows_are_convex_combinations_of_supported_values():
+    """Abar rows are distributions over the supported admissible keys: with V
+    = one-hot columns marking whether a key is supported, O sums to 1 on the
+    supported column and 0 elsewhere."""
+    B, H, Hkv, L, D, blk = 1, 2, 1, 32, 4, 8
+    Q, K, _ = synth.random_qkv(B, H, Hkv, L, D, seed=25)
+    idx, counts = synth.random_support(B, Hkv, L // blk, 2, seed=26)
+    # For the rows of query block q: V column 0 marks the keys whose block is
+    # in q's support, column 1 the others.
+    got_rows = []
+    for q in range(L // blk):
+        inside = np.zeros((B, Hkv, L, 2))
+        sup = set(int(v) for v in idx[0, 0, q, :counts[0, 0, q]])
+        for j in range(L):
+            inside[0, 0, j, 0 if j // blk in sup else 1] = 1.0
+        O = orc.freeze_a(bf16_vals(Q), bf16_vals(K), inside, idx, counts, blk)
+        got_rows.append(O[0, :, q * blk:(q + 1) * blk, :])
+    got = np.stack(got_rows)
+    np.testing.assert_allclose(got[..., 0], 1.0, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(got[..., 1], 0.0, rtol=0, atol=1e-12)
