@@ -450,6 +450,43 @@ def main():
     torch.cuda.synchronize()
     freeze_a_ms = statistics.mean(a.elapsed_time(b) for a, b in fz_ev)
 
+    # ---- the paper's default block of 32 keys: the 4K workload at B = 32 with
+    # the same key budget per query block, its own discovery and selection,
+    # then late steps timed.  Kernels compute 128 x 128 tiles with 4 x 4
+    # sub-block masks, so `tile_density` (tiles touched / causal tiles) is the
+    # share of tensor work against the dense kernel.
+    wl32 = synth.WORKLOADS["4k_b32"]
+    shape32, sel32 = wise.shape_of(wl32), wise.select_of(wl32)
+    layer32 = wise.WiseAttention(shape32, sel32, wl32.n_discovery)
+    traj32 = synth.Trajectory(wl32)
+    late32 = 8
+    steps32 = [tuple(torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).cuda() for x in traj32.step(t))
+               for t in range(wl32.n_discovery + late32)]
+    O32 = torch.empty_like(steps32[0][0])
+    for t in range(wl32.n_discovery + 1):
+        layer32.step(t, *steps32[t], O32)
+    ev32 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(late32)]
+    for rep in range(2):  # the first pass warms up
+        for i, t in enumerate(range(wl32.n_discovery, wl32.n_discovery + late32)):
+            ev32[i][0].record(stream)
+            wise.wise_sparse_attn(shape32, *steps32[t], layer32.idx, layer32.counts, O32)
+            ev32[i][1].record(stream)
+        torch.cuda.synchronize()
+    b32_ms = statistics.mean(a.elapsed_time(b) for a, b in ev32)
+    i32, c32 = layer32.idx.cpu().numpy(), layer32.counts.cpu().numpy()
+    f32 = sparse_flops(i32, c32, wl32.n_heads, wl32.head_dim, wl32.block)
+    tiles32 = 0
+    for b in range(wl32.batch):
+        for g in range(wl32.n_kv_heads):
+            for qt in range(wl32.n_blocks // 4):
+                tiles32 += len({int(v) // 4 for q in range(4 * qt, 4 * qt + 4) for v in i32[b, g, q, :c32[b, g, q]]})
+    causal_tiles = wl32.batch * wl32.n_kv_heads * (wl32.seqlen // 128) * (wl32.seqlen // 128 + 1) // 2
+    block32 = {"workload": "4k_b32: the 4K workload at block 32, sink+diagonal+95% coverage cap 32",
+               "late_ms": round(b32_ms, 5), "tflops_effective": round(f32 / (b32_ms * 1e-3) / 1e12, 2),
+               "density": round(f32 / dense_flops(wl32.batch, wl32.n_heads, wl32.seqlen, wl32.head_dim), 4),
+               "tile_density": round(tiles32 / causal_tiles, 4), "speedup_vs_dense": round(statistics.mean(dense_ms) / b32_ms, 4)}
+    del steps32, layer32, O32
+
     # ---- the whole trajectory as one CUDA graph (discovery, selection, late
     # steps), replayed; its launches carry no host-side gaps
     graph = {"ms": None, "note": None}
@@ -520,6 +557,7 @@ def main():
         "block_density": round(float(layer.counts.sum()) / (wl.batch * wl.n_kv_heads * nb * (nb + 1) / 2), 4),
         "supports": supports,
         "rolling_jaccard_at_discovery_end": round(rolling_jaccard, 4),
+        "block32": block32,
         "freeze_a_ms": round(freeze_a_ms, 5),
         "all_blocks_vs_dense": round(all_blocks_ms / dense, 4),
         "graph_trajectory_ms": None if graph["ms"] is None else round(graph["ms"], 4),

@@ -17,8 +17,10 @@
  *    [batch, n_kv_heads, seqlen, head_dim] bf16.  Query head h reads kv-head
  *    h / (n_heads / n_kv_heads) (grouped-query attention).
  *  - Q/K/V/O must be 16-byte aligned, blockmass/idx/counts 4-byte aligned.
- *  - head_dim is 64, 96 or 128; block (B) is 64 or 128; seqlen % block == 0.
- *    nQB = nKB = seqlen / block.
+ *  - head_dim is 64, 96 or 128; block (B) is 32 (the paper's default, Sec.
+ *    5.1), 64 or 128; seqlen % block == 0.  nQB = nKB = seqlen / block.  The
+ *    attention kernels compute 128 x 128 tiles whatever B is: a smaller block
+ *    is a sub-block of a tile, masked per (query block, key block) pair.
  *  - Every call is asynchronous on `stream` and returns a status code
  *    (WISE_OK or a negative WISE_ERR_*) describing argument checks and the
  *    launch; nothing is done when a check fails.  Faults found by a kernel
@@ -123,11 +125,11 @@ int wise_full_attn_accumulate(const wise_shape_t* shape, const void* Q, const vo
  *
  * Arguments, layouts and results are those of wise_full_attn_accumulate;
  * blockmass must not be NULL (plain dense attention uses no scratch).
- * Limit: one call needs min(batch*n_heads*ceil(seqlen/128), SM count) *
- * (2048 * (nKB/2 + 1) + 64 * nKB) bytes of scratch (nKB/2 rounded down);
- * larger problems return WISE_ERR_UNSUPPORTED and launch nothing.  On a
- * 152-SM GB300 with at least 152 query tiles that is nKB <= 49 (seqlen <=
- * 6272 with block 128).
+ * Limit: with nT = ceil(seqlen/128) tiles and S = 128/block, one call needs
+ * min(batch*n_heads*nT, SM count) * (2048 * S * (nT/2 + 1) + 64 * nKB)
+ * bytes of scratch (nT/2 rounded down); larger problems return
+ * WISE_ERR_UNSUPPORTED and launch nothing.  On a 152-SM GB300 with at least
+ * 152 query tiles that is nT <= 49 with block 128 (seqlen <= 6272).
  * The first call on each device looks up the array's device address (with
  * that device current) and caches it; make that first call before any CUDA
  * stream capture.  All calls on a device share the one array: calls whose
@@ -201,7 +203,8 @@ int wise_support_mass(const wise_shape_t* shape, const float* blockmass, const i
  * first counts entries are used; they must be ascending block ids in
  * [0, q].  Entries that break this are skipped and flagged as
  * WISE_ERR_BAD_SUPPORT in the status word.  A query row with no admissible key
- * gets O = 0. */
+ * gets O = 0.  cap <= 0 is WISE_ERR_INVALID_ARG, cap > 65535
+ * WISE_ERR_UNSUPPORTED. */
 int wise_sparse_attn(const wise_shape_t* shape, const void* Q, const void* K, const void* V, const int32_t* idx,
                      const int32_t* counts, int cap, void* O, cudaStream_t stream);
 

@@ -9,15 +9,17 @@
 // grid (one CTA per SM) deals them out in a snake order (CTA c takes unit
 // k*G + c in even rounds k and k*G + G-1-c in odd rounds), which evens out
 // the per-CTA sums of the decreasing lengths.  Each unit walks its list of
-// key tiles (BN keys each): every tile of the causal prefix (dense), or the
-// blocks of the support (sparse; with block 64 a query tile covers two query
-// blocks and walks the union of their lists, masking per half).
+// key tiles (128 keys each): every tile of the causal prefix (dense), or the
+// tiles holding blocks of the support (sparse).  With a block B of 32 or 64 a
+// query tile covers S = 128 / B query blocks and a key tile S key blocks; the
+// unit walks the union of its query blocks' lists, and each tile carries an
+// S x S mask of the (query block, key block) pairs that attend.
 //
-// Both products run with the A operand in tensor memory, because a tcgen05
-// MMA that reads both operands from shared memory is limited by the shared
-// memory read rate to about half the tensor peak (measured: 118 clk per
-// M128/N128/K16 step with both operands in shared memory, 66 clk with A in
-// TMEM):
+// Both products run with the A operand in tensor memory: Q is copied into
+// TMEM once per unit, so that its staging buffer can already receive the next
+// unit's Q.  (With two threads issuing, MMAs with A in shared memory run at
+// the same rate; one thread alone issues at most about one MMA per 89 clk
+// against the 64 clk an M128/N128/K16 step takes, hence two issuers.)
 //   S = Q K^T    Q copied per unit from shared memory into TMEM with
 //                tcgen05.cp (ordered before the MMAs that read it), K from
 //                shared memory (K-major);
@@ -79,11 +81,17 @@
 
 namespace wise {
 
-template <int D, int BN>
+// Key tiles are 128 keys wide whatever the block size: a tcgen05 MMA issued by
+// one thread costs about the same issue time at N = 32, 64 or 128, so narrower
+// tiles only waste tensor throughput.  Blocks of 32 or 64 are sub-blocks of a
+// tile, selected per (query block, key block) by the tile's mask.
+constexpr int kTileN = 128;
+
+template <int D>
 struct AttnCfg {
   static constexpr int kBoxes = (D + 63) / 64;          // 64-column TMA boxes per row tile
   static constexpr int kQBytes = kBoxes * 128 * 128;    // one 128-row Q tile (staging)
-  static constexpr int kKVBytes = kBoxes * BN * 128;    // one BN-row K or V tile (one ring entry)
+  static constexpr int kKVBytes = kBoxes * kTileN * 128; // one 128-row K or V tile (one ring entry)
   // Static shared memory (barriers, schedule ring, row exchange buffers).
   static constexpr int kStaticReserve = 7 * 1024;
   // Dynamic shared memory available after the 1024-byte alignment slack.
@@ -115,15 +123,16 @@ struct AttnCfg {
   static constexpr int kMmaSWarp = 9;   // issues S = Q K^T, owns the TMEM allocation
   static constexpr int kMmaPVWarp = 10; // issues O += P V
   static_assert(kRingV >= 1 && kRingK >= 2, "shared memory budget");
-  static_assert(BN <= 128 && D <= 128, "TMEM budget");
+  static_assert(D <= 128, "TMEM budget");
   static_assert(256 * kRegsSoftmax + 128 * kRegsOther <= kThreads * 168, "register split");
 };
 
-// Tile schedule rings.  Entry = {key block, unit, flags, tile index within
-// its unit} (for the end marker: {0, 0, kEntEnd, number of tiles}).  The low
-// two flag bits say which 64-row halves of the query tile attend the key
-// block; bits 8 and up hold the index of the unit among this CTA's units
-// with tiles.
+// Tile schedule rings.  Entry = {key tile | mask << 16, unit, flags, tile
+// index within its unit} (for the end marker: {0, 0, kEntEnd, number of
+// tiles}).  With S = 128 / block query blocks per query tile and key blocks
+// per key tile, bit qi * S + ki of the mask says that query block qi of the
+// tile attends key block ki of the key tile.  Flag bits 8 and up hold the
+// index of the unit among this CTA's units with tiles.
 constexpr int kSchedSlots = 16;  // per ring
 constexpr int kEntFirst = 4;     // first tile of its unit
 constexpr int kEntLast = 8;      // last tile of its unit
@@ -184,61 +193,86 @@ __device__ __forceinline__ float exp2_scaled(float (&s)[N], float scale, float s
   return b.x + b.y;
 }
 
-// Key tiles of one unit in ascending order.  Dense: 0..last.  Sparse: the
-// support list of the unit's query block (block 128), or the merge of the
-// lists of its two query blocks (block 64); `bits` says which half of the
-// 128 query rows may attend the tile.  Entries that are negative, beyond the
-// query block, or not strictly ascending are skipped and flagged in `bad`.
-// Fields a variant does not use are never touched, so they cost no registers.
-template <int BN, int MODE>
+// exp2_scaled that also returns the sums of the S column groups of N / S
+// columns (the key sub-blocks of a tile), for the block masses; S = 2 or 4.
+template <int N, int S>
+__device__ __forceinline__ float exp2_scaled_groups(float (&s)[N], float scale, float shift, float (&g)[S]) {
+  static_assert(S == 2 || S == 4, "groups");
+  constexpr int kChains = 4 / S;  // independent accumulation chains per group
+  constexpr int kCols = N / S;
+  const float2 sc = make_float2(scale, scale), sh = make_float2(-shift, -shift);
+  float2 acc[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) acc[e] = make_float2(0.0f, 0.0f);
+#pragma unroll
+  for (int c = 0; c < N; c += 2) {
+    const float2 x = __ffma2_rn(make_float2(s[c], s[c + 1]), sc, sh);
+    const float2 y = make_float2(ex2_approx(x.x), ex2_approx(x.y));
+    s[c] = y.x;
+    s[c + 1] = y.y;
+    const int a = (c / kCols) * kChains + (c / 2) % kChains;
+    acc[a] = __fadd2_rn(acc[a], y);
+  }
+  float total = 0.0f;
+#pragma unroll
+  for (int k = 0; k < S; ++k) {
+    float2 t = acc[k * kChains];
+#pragma unroll
+    for (int ch = 1; ch < kChains; ++ch) t = __fadd2_rn(t, acc[k * kChains + ch]);
+    g[k] = t.x + t.y;
+    total += g[k];
+  }
+  return total;
+}
+
+// Key tiles of one unit in ascending order, with their sub-block masks
+// (S = 128 / BLK).  Dense: tiles 0..last, every sub-block (the causal limit is
+// applied per row).  Sparse: the merge of the support lists of the unit's S
+// query blocks; key block kb lies in key tile kb / S.  Entries that are
+// negative, beyond their query block, or not strictly ascending are skipped
+// and flagged in `bad`.  Fields a variant does not use are never touched, so
+// they cost no registers.
+template <int BLK, int MODE>
 struct TileIter {
-  int cur, last;                                   // dense
-  const int32_t* la;                               // sparse, first query block
-  int na, ia, lima, preva, pend_a;
-  const int32_t* lb;                               // sparse, second query block (block 64)
-  int nb, ib, limb, prevb, pend_b;
+  static constexpr int S = kTileN / BLK;
+  int cur, last;             // dense
+  const int32_t* l0;         // sparse: list of query block q0; list q at l0 + q * cap
+  int cap, q0;
+  int pos[S];                // list q: entries read (low 16 bits) and count (high 16 bits); cap < 2^16
+  int pend[S];               // next entry of list q (the last one accepted), INT_MAX when done
   int bad;
 
-  __device__ __forceinline__ int pull(const int32_t* l, int n, int& i, int lim, int& prev) {
-    while (i < n) {
-      const int v = __ldg(l + i);
-      ++i;
-      if (v >= 0 && v <= lim && v > prev) {
-        prev = v;
-        return v;
-      }
+  // Next valid entry of list q after pend[q]: in [0, q0 + q] and above it.
+  __device__ __forceinline__ int pull(int q) {
+    const int prev = pend[q];
+    while ((pos[q] & 0xFFFF) < (pos[q] >> 16)) {
+      const int v = __ldg(l0 + (size_t)q * cap + (pos[q] & 0xFFFF));
+      ++pos[q];
+      if (v >= 0 && v <= q0 + q && v > prev) return v;
       bad = 1;
     }
     return INT_MAX;
   }
 
-  __device__ __forceinline__ bool next(int& kb, int& bits) {
+  __device__ __forceinline__ bool next(int& kt, uint32_t& mask) {
     if constexpr (MODE != kSparse) {
       if (cur > last) return false;
-      kb = cur++;
-      bits = 3;
-      return true;
-    } else if constexpr (BN == 128) {
-      if (pend_a == INT_MAX) return false;
-      kb = pend_a;
-      bits = 1;
-      pend_a = pull(la, na, ia, lima, preva);
+      kt = cur++;
+      mask = S == 1 ? 1u : S == 2 ? 0xFu : 0xFFFFu;
       return true;
     } else {
-      if (pend_a == INT_MAX && pend_b == INT_MAX) return false;
-      if (pend_a < pend_b) {
-        kb = pend_a;
-        bits = 1;
-        pend_a = pull(la, na, ia, lima, preva);
-      } else if (pend_b < pend_a) {
-        kb = pend_b;
-        bits = 2;
-        pend_b = pull(lb, nb, ib, limb, prevb);
-      } else {
-        kb = pend_a;
-        bits = 3;
-        pend_a = pull(la, na, ia, lima, preva);
-        pend_b = pull(lb, nb, ib, limb, prevb);
+      int lo = pend[0];
+#pragma unroll
+      for (int q = 1; q < S; ++q) lo = min(lo, pend[q]);
+      if (lo == INT_MAX) return false;
+      kt = lo / S;
+      mask = 0;
+#pragma unroll
+      for (int q = 0; q < S; ++q) {
+        while (pend[q] != INT_MAX && pend[q] / S == kt) {
+          mask |= 1u << (q * S + pend[q] % S);
+          pend[q] = pull(q);
+        }
       }
       return true;
     }
@@ -253,32 +287,28 @@ __device__ __forceinline__ int clamp_count(int n, int cap, int& bad) {
   return n;
 }
 
-template <int BN, int MODE>
-__device__ __forceinline__ TileIter<BN, MODE> make_iter(const AttnParams& p, int b, int kvh, int qt) {
-  TileIter<BN, MODE> it;
+template <int BLK, int MODE>
+__device__ __forceinline__ TileIter<BLK, MODE> make_iter(const AttnParams& p, int b, int kvh, int qt) {
+  TileIter<BLK, MODE> it;
   it.bad = 0;
   if constexpr (MODE != kSparse) {
     it.cur = 0;
     const int last_row = min(qt * 128 + 127, p.seqlen - 1);
-    it.last = last_row / BN;
+    it.last = last_row / kTileN;
   } else {
-    constexpr int kQbPerTile = 128 / BN;
-    const int q0 = qt * kQbPerTile;
+    constexpr int S = TileIter<BLK, MODE>::S;
+    const int q0 = qt * S;
     const size_t row0 = ((size_t)b * p.n_kv_heads + kvh) * p.n_blocks + q0;
-    it.la = p.idx + row0 * p.cap;
-    it.na = clamp_count(__ldg(p.counts + row0), p.cap, it.bad);
-    it.ia = 0;
-    it.lima = q0;
-    it.preva = -1;
-    it.pend_a = it.pull(it.la, it.na, it.ia, it.lima, it.preva);
-    if constexpr (kQbPerTile == 2) {
-      it.lb = p.idx + (row0 + 1) * p.cap;
-      it.nb = (q0 + 1 < p.n_blocks) ? clamp_count(__ldg(p.counts + row0 + 1), p.cap, it.bad) : 0;
-      it.ib = 0;
-      it.limb = q0 + 1;
-      it.prevb = -1;
-      it.pend_b = it.pull(it.lb, it.nb, it.ib, it.limb, it.prevb);
+    it.l0 = p.idx + row0 * p.cap;
+    it.cap = p.cap;
+    it.q0 = q0;
+#pragma unroll
+    for (int q = 0; q < S; ++q) {
+      it.pos[q] = ((q0 + q < p.n_blocks) ? clamp_count(__ldg(p.counts + row0 + q), p.cap, it.bad) : 0) << 16;
+      it.pend[q] = -1;
     }
+#pragma unroll
+    for (int q = 0; q < S; ++q) it.pend[q] = it.pull(q);
   }
   return it;
 }
@@ -334,11 +364,11 @@ __device__ __forceinline__ void raise_status(const AttnParams& p, int* abort, in
 }
 
 // ------------------------------------------------------------------ producer
-template <int D, int BN, int MODE>
+template <int D, int BLK, int MODE>
 __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, const CUtensorMap* mapV,
                               const AttnParams& p, uint8_t* q_stage, uint8_t* ring,
-                              SharedState<AttnCfg<D, BN>::kRingK, AttnCfg<D, BN>::kRingV>& sb) {
-  using C = AttnCfg<D, BN>;
+                              SharedState<AttnCfg<D>::kRingK, AttnCfg<D>::kRingV>& sb) {
+  using C = AttnCfg<D>;
   constexpr int RK = C::kRingK, RV = C::kRingV;
   uint8_t* k_ring = ring;
   uint8_t* v_ring = ring + RK * C::kKVBytes;
@@ -365,7 +395,7 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
     if (j >= R && !mbar_wait(&empty[slot], ((j / R) - 1) & 1, abort)) return false;
     mbar_arrive_expect_tx(&full[slot], C::kKVBytes);
     for (int i = 0; i < C::kBoxes; ++i)
-      tma_load_3d(base + slot * C::kKVBytes + i * BN * 128, map, &full[slot], 64 * i, kb * BN, z);
+      tma_load_3d(base + slot * C::kKVBytes + i * kTileN * 128, map, &full[slot], 64 * i, kb * kTileN, z);
     ++j;
     return true;
   };
@@ -379,9 +409,10 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
     decode_unit(p, u, b, h, qt);
     const int kvh = h / p.group;
     const int z = b * p.n_kv_heads + kvh;
-    auto it = make_iter<BN, MODE>(p, b, kvh, qt);
-    int kb, bits;
-    bool have = it.next(kb, bits);
+    auto it = make_iter<BLK, MODE>(p, b, kvh, qt);
+    int kb;
+    uint32_t mask;
+    bool have = it.next(kb, mask);
     if (!have) {
       if (!emit(0, 0, u, kEntEmpty, 0)) ok = false;
       ++n_empty;
@@ -389,10 +420,12 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
     bool first = true;
     const int unit_ix = nq;  // index of this unit among the units with tiles
     for (int t = 0; have && ok; ++t) {
-      int nkb, nbits;
-      const bool more = it.next(nkb, nbits);
-      const int flags = bits | (first ? kEntFirst : 0) | (more ? 0 : kEntLast) | (unit_ix << kEntUnitShift);
-      if (!emit(kMmaRing, kb, u, flags, t) || !emit(jt & 1, kb, u, flags, t)) {
+      int nkb;
+      uint32_t nmask;
+      const bool more = it.next(nkb, nmask);
+      const int flags = (first ? kEntFirst : 0) | (more ? 0 : kEntLast) | (unit_ix << kEntUnitShift);
+      const int key = (int)((uint32_t)kb | (mask << 16));
+      if (!emit(kMmaRing, key, u, flags, t) || !emit(jt & 1, key, u, flags, t)) {
         ok = false;
         break;
       }
@@ -420,7 +453,7 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
       prev_z = z;
       have_prev = true;
       kb = nkb;
-      bits = nbits;
+      mask = nmask;
       have = more;
       first = false;
     }
@@ -452,13 +485,13 @@ __device__ __forceinline__ bool sched_read_mma(SS& sb, int e, int4& ent, volatil
 }
 
 // --------------------------------------------------------------- MMA issuers
-template <int D, int BN, int MODE>
+template <int D, int BLK, int MODE>
 __device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* q_stage, uint8_t* ring,
-                           SharedState<AttnCfg<D, BN>::kRingK, AttnCfg<D, BN>::kRingV>& sb) {
-  using C = AttnCfg<D, BN>;
+                           SharedState<AttnCfg<D>::kRingK, AttnCfg<D>::kRingV>& sb) {
+  using C = AttnCfg<D>;
   constexpr int RK = C::kRingK;
   volatile int* abort = &sb.abort;
-  constexpr uint32_t idesc_s = idesc_bf16_f32(128, BN, false, false);
+  constexpr uint32_t idesc_s = idesc_bf16_f32(128, kTileN, false, false);
   int j = 0, nq = 0;
   bool ok = true;
   for (;;) {
@@ -504,7 +537,7 @@ __device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* q_stage,
     for (int kk = 0; kk < D / 16; ++kk) {
       // K step kk: 8 TMEM columns of Q; shared-memory descriptors of later
       // steps differ only in the start address field (address >> 4).
-      const uint32_t b_off = ((kk >> 2) * (BN * 128) + (kk & 3) * 32) >> 4;
+      const uint32_t b_off = ((kk >> 2) * (kTileN * 128) + (kk & 3) * 32) >> 4;
       umma_bf16_ts(tmem + s_col, tmem + C::kTmemQ + kk * 8, b0 + b_off, idesc_s, kk > 0 ? 1u : 0u);
     }
     umma_commit(&sb.s_full[j & 1]);
@@ -519,10 +552,10 @@ __device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* q_stage,
   mbar_wait(&sb.s_done, 0, &never);
 }
 
-template <int D, int BN, int MODE>
+template <int D, int BLK, int MODE>
 __device__ void attn_mma_pv(const AttnParams& p, uint32_t tmem, uint8_t* ring,
-                            SharedState<AttnCfg<D, BN>::kRingK, AttnCfg<D, BN>::kRingV>& sb) {
-  using C = AttnCfg<D, BN>;
+                            SharedState<AttnCfg<D>::kRingK, AttnCfg<D>::kRingV>& sb) {
+  using C = AttnCfg<D>;
   constexpr int RK = C::kRingK, RV = C::kRingV;
   uint8_t* v_ring = ring + RK * C::kKVBytes;
   volatile int* abort = &sb.abort;
@@ -557,9 +590,9 @@ __device__ void attn_mma_pv(const AttnParams& p, uint32_t tmem, uint8_t* ring,
     }
     tc_fence_after_sync();
     const uint32_t p_col = C::kTmemP + (j & 1) * C::kTmemPCols;
-    const uint64_t b0 = smem_desc_sw128(smem_u32(v_ring + slot * C::kKVBytes), BN * 128, 1024);
+    const uint64_t b0 = smem_desc_sw128(smem_u32(v_ring + slot * C::kKVBytes), kTileN * 128, 1024);
 #pragma unroll 1
-    for (int kk = 0; kk < BN / 16; ++kk)
+    for (int kk = 0; kk < kTileN / 16; ++kk)
       umma_bf16_ts(tmem + C::kTmemO, tmem + p_col + kk * 8, b0 + ((kk * 2048) >> 4), idesc_o,
                    (first && kk == 0) ? 0u : 1u);
     umma_commit(&sb.o_full[j & 1]);
@@ -594,17 +627,22 @@ __device__ __forceinline__ void tmem_load_row(uint32_t addr, float (&x)[N]) {
   }
 }
 
-// Loads this thread's row of an S tile (kCols columns) and applies the
-// causal / support masks.
-template <int kCols>
-__device__ __forceinline__ void load_s_row(uint32_t addr, float (&s)[kCols], bool attend, int lim) {
-  tmem_load_row<kCols>(addr, s);
-  // Keys with column c > lim are in the future of this row; a row that does
-  // not attend the tile masks every column.
-  const int lim_eff = attend ? lim : -1;
-  if (lim_eff < kCols - 1) {
+// Loads this thread's row of an S tile (kTileN columns) and applies the
+// causal / support masks: column c of key sub-block k = c / BLK is kept if
+// bit k of `sub` is set and c <= lim (keys with c > lim are in the future of
+// this row).
+template <int BLK>
+__device__ __forceinline__ void load_s_row(uint32_t addr, float (&s)[kTileN], uint32_t sub, int lim) {
+  constexpr int S = kTileN / BLK;
+  tmem_load_row<kTileN>(addr, s);
+  if (sub != (1u << S) - 1u || lim < kTileN - 1) {
+    // Per sub-block limit: lim where the row attends the sub-block, else the
+    // column before it, so that a single compare masks the column.
+    int lim_k[S];
 #pragma unroll
-    for (int c = 0; c < kCols; ++c) s[c] = (c > lim_eff) ? -INFINITY : s[c];
+    for (int k = 0; k < S; ++k) lim_k[k] = ((sub >> k) & 1u) ? lim : k * BLK - 1;
+#pragma unroll
+    for (int c = 0; c < kTileN; ++c) s[c] = (c > lim_k[c / BLK]) ? -INFINITY : s[c];
   }
 }
 
@@ -619,10 +657,10 @@ struct EpiInfo {
 };
 
 // ------------------------------------------------------------------- softmax
-template <int D, int BN, int MODE>
+template <int D, int BLK, int MODE>
 __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w, uint32_t tmem, uint8_t* out_stage,
-                             SharedState<AttnCfg<D, BN>::kRingK, AttnCfg<D, BN>::kRingV>& sb) {
-  using C = AttnCfg<D, BN>;
+                             SharedState<AttnCfg<D>::kRingK, AttnCfg<D>::kRingV>& sb) {
+  using C = AttnCfg<D>;
   constexpr float kRescaleThreshold = 8.0f;   // log2 units: P stays <= 256
   volatile int* abort = &sb.abort;
   const int r = threadIdx.x & 127;  // query row within the tile (TMEM lane)
@@ -630,17 +668,18 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
   const uint32_t lane_tmem = tmem + ((uint32_t)(wq * 32) << 16);
   const uint32_t s_col = C::kTmemS;
   const uint32_t p_col = C::kTmemP + w * C::kTmemPCols;  // this warpgroup's P buffer
-  const int half_bit = (BN == 64) ? (1 << (r >> 6)) : 1;
+  constexpr int S = kTileN / BLK;   // query blocks per query tile = key blocks per key tile
+  const int qsub = r / BLK;         // this row's query block within the tile
   // Per-CTA scratch (kDenseMass): log2 partial masses [2 warpgroups][2 units]
-  // [n_blocks / 2 + 1 tiles][128 rows] (tile t of a unit sits at t / 2 in
-  // the region of the warpgroup that handled it), then [2 warpgroups][2]
-  // [4 warps][n_blocks] per-warp column sums.
-  const int lc_tiles = p.n_blocks / 2 + 1;
-  float* cta_scratch = p.scratch + (size_t)blockIdx.x * scratch_floats_per_cta(p.n_blocks);
-  auto lc_at = [&](int g, int unit, int t) -> float* {
-    return cta_scratch + ((size_t)(g * 2 + (unit & 1)) * lc_tiles + (t >> 1)) * 128 + r;
+  // [key tiles / 2 + 1][S sub-blocks][128 rows] (tile t of a unit sits at
+  // t / 2 in the region of the warpgroup that handled it), then
+  // [2 warpgroups][2][4 warps][n_blocks] per-warp column sums.
+  const int lc_tiles = p.n_qtiles / 2 + 1;
+  float* cta_scratch = p.scratch + (size_t)blockIdx.x * scratch_floats_per_cta(p.n_qtiles, S, p.n_blocks);
+  auto lc_at = [&](int g, int unit, int t, int k) -> float* {
+    return cta_scratch + (((size_t)(g * 2 + (unit & 1)) * lc_tiles + (t >> 1)) * S + k) * 128 + r;
   };
-  float* warp_sums = cta_scratch + (size_t)4 * lc_tiles * 128;
+  float* warp_sums = cta_scratch + (size_t)4 * lc_tiles * S * 128;
 
   int j = w;             // this warpgroup's next tile: w, w + 2, ...
   int pos = 0;           // entries read from ring w
@@ -651,14 +690,16 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
   float l_w = 0.0f, m_w = -INFINITY;  // this warpgroup's part of the row sum, relative to m_w
   bool ok = true;
 
-  // ---- one tile (j & 1 == w): key block kb, tile t of the unit with index unit_ix
-  auto tile = [&](int kb, int bits, bool first, int t, int unit_ix) -> bool {
+  // ---- one tile (j & 1 == w): key tile and mask in `key`, tile t of the
+  // unit with index unit_ix
+  auto tile = [&](int key, bool first, int t, int unit_ix) -> bool {
     if (!warp_wait(&sb.s_full[w], (j >> 1) & 1, abort)) return false;
     tc_fence_after_sync();
-    const bool attend = (bits & half_bit) != 0;
-    const int lim = cur_row - kb * BN;  // keys kb*BN + c with c > lim are in the future
-    float s[BN];
-    load_s_row<BN>(lane_tmem + s_col, s, attend, lim);
+    const int kb = key & 0xFFFF;
+    const uint32_t sub = ((uint32_t)key >> (16 + qsub * S)) & ((1u << S) - 1u);
+    const int lim = cur_row - kb * kTileN;  // keys kb*128 + c with c > lim are in the future
+    float s[kTileN];
+    load_s_row<BLK>(lane_tmem + s_col, s, sub, lim);
     // S(j) is in registers: S(j+1) may overwrite it.
     tc_fence_before_sync();
     __syncwarp();
@@ -675,18 +716,25 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     sb.mx[w][(j >> 1) & 1][r] = m_new;
     __syncwarp();
     if (lane == 0) mbar_arrive(&sb.m_pub[w][(j >> 1) & 1]);
-    const float rowsum = exp2_scaled(s, p.scale_log2, m_new == -INFINITY ? 0.0f : m_new);
+    float gsum[S];  // kDenseMass: sums of p over the key sub-blocks
+    float rowsum;
+    if constexpr (MODE == kDenseMass && S > 1) {
+      rowsum = exp2_scaled_groups(s, p.scale_log2, m_new == -INFINITY ? 0.0f : m_new, gsum);
+    } else {
+      rowsum = exp2_scaled(s, p.scale_log2, m_new == -INFINITY ? 0.0f : m_new);
+      gsum[0] = rowsum;
+    }
     // P as bf16 pairs, packed before the wait below.
-    uint32_t pw[BN / 2];
+    uint32_t pw[kTileN / 2];
 #pragma unroll
-    for (int e = 0; e < BN / 2; ++e) pw[e] = pack_bf16x2(s[2 * e], s[2 * e + 1]);
+    for (int e = 0; e < kTileN / 2; ++e) pw[e] = pack_bf16x2(s[2 * e], s[2 * e + 1]);
     // P buffer w was last read by P V(j-2); this warpgroup waited for P V(j-4)
     // at its previous tile, so o_full[w] is at most one phase short.
     if (j >= 2 && !warp_wait(&sb.o_full[w], ((j >> 1) - 1) & 1, abort)) return false;
     tc_fence_after_sync();
     // The stores complete while the bookkeeping below runs.
 #pragma unroll
-    for (int c = 0; c < BN / 32; ++c) {
+    for (int c = 0; c < kTileN / 32; ++c) {
       uint32_t q[16];
 #pragma unroll
       for (int e = 0; e < 16; ++e) q[e] = pw[16 * c + e];
@@ -701,7 +749,11 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     // other warpgroup after any epilogue it ran for unit unit_ix - 2 (which
     // read this slot), and this warpgroup's own epilogues precede in program
     // order.
-    if (MODE == kDenseMass) *lc_at(w, unit_ix, t) = rowsum > 0.0f ? m_new + lg2_approx(rowsum) : -INFINITY;
+    if constexpr (MODE == kDenseMass) {
+#pragma unroll
+      for (int k = 0; k < S; ++k)
+        *lc_at(w, unit_ix, t, k) = gsum[k] > 0.0f ? m_new + lg2_approx(gsum[k]) : -INFINITY;
+    }
     // O (after P V(j-1)) is rescaled only when the max moved.  tcgen05.ld/st
     // are warp-collective: the warp rescales together, lanes whose max did
     // not move use a factor of 1.
@@ -780,36 +832,33 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
       // each query block.  E wrote its tiles' lc before publishing its part.
       const float lse = ei.m + lg2_approx(l_row);
       float* ws = warp_sums + (size_t)(w * 2 + (n_epi & 1)) * 4 * p.n_blocks;
-      const int n_kt = ei.n_kt;
-      // Dense variants: tile t of the unit is key block t.
-      for (int t = 0; t < n_kt; ++t) {
-        const float lc = *lc_at((ei.j0 + t) & 1, ei.nu, t);
+      // Dense variants: tile t of the unit is key tile t, holding key blocks
+      // t * S .. t * S + S - 1.
+      const int n_kb = min(ei.n_kt * S, p.n_blocks);
+      for (int kb = 0; kb < n_kb; ++kb) {
+        const int t = kb / S;
+        const float lc = *lc_at((ei.j0 + t) & 1, ei.nu, t, kb - t * S);
         float v = (row < p.seqlen) ? ex2_approx(lc - lse) : 0.0f;
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-        if (lane == 0) ws[wq * p.n_blocks + t] = v;
+        if (lane == 0) ws[wq * p.n_blocks + kb] = v;
       }
       // Orders the four warps' writes before the reads below (release /
       // acquire at CTA scope).
       __syncwarp();
       if (lane == 0) mbar_arrive(&sb.epi[w]);
       if (!warp_wait(&sb.epi[w], n_epi & 1, abort)) return false;
-      constexpr int kHalves = 128 / BN;  // query blocks per tile
-      const float inv_b = 1.0f / (float)BN;
-      for (int e = r; e < kHalves * p.n_blocks; e += 128) {
-        const int hf = e / p.n_blocks, t = e % p.n_blocks;
-        const int qblock = qt * kHalves + hf;
+      constexpr int kWarpsPerBlock = BLK / 32;  // warps holding one query block's rows
+      const float inv_b = 1.0f / (float)BLK;
+      for (int e = r; e < S * p.n_blocks; e += 128) {
+        const int qi = e / p.n_blocks, kb = e % p.n_blocks;
+        const int qblock = qt * S + qi;
         if (qblock >= p.n_blocks) continue;
-        float* out = p.blockmass + ((size_t)(b * p.n_heads + h) * p.n_blocks + qblock) * p.n_blocks + t;
-        if (t < n_kt) {
+        float* out = p.blockmass + ((size_t)(b * p.n_heads + h) * p.n_blocks + qblock) * p.n_blocks + kb;
+        if (kb < n_kb) {
           float sum = 0.0f;
-          if (BN == 128) {
 #pragma unroll
-            for (int q = 0; q < 4; ++q) sum += ws[q * p.n_blocks + t];
-          } else {
-#pragma unroll
-            for (int q = 2 * hf; q < 2 * hf + 2; ++q) sum += ws[q * p.n_blocks + t];
-          }
+          for (int q = qi * kWarpsPerBlock; q < (qi + 1) * kWarpsPerBlock; ++q) sum += ws[q * p.n_blocks + kb];
           sum *= inv_b;
           *out = (p.step == 0) ? sum : *out + sum;
         } else if (p.step == 0) {
@@ -879,14 +928,14 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
       l_w = 0.0f;
       m_w = -INFINITY;
     }
-    if (!tile(ent.x, fl & 3, first, ent.w, fl >> kEntUnitShift)) {
+    if (!tile(ent.x, first, ent.w, fl >> kEntUnitShift)) {
       ok = false;
       break;
     }
     fresh = false;
     if (fl & kEntLast) {
       // L: this warpgroup handled the unit's last tile.
-      const EpiInfo ei{ent.y, j - ent.w, j, fl >> kEntUnitShift, ent.x + 1, l_w, m_w};
+      const EpiInfo ei{ent.y, j - ent.w, j, fl >> kEntUnitShift, (ent.x & 0xFFFF) + 1, l_w, m_w};
       if (!epilogue(ei)) {
         ok = false;
         break;
@@ -901,12 +950,12 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
 }
 
 // -------------------------------------------------------------------- kernel
-template <int D, int BN, int MODE>
-__global__ void __launch_bounds__(AttnCfg<D, BN>::kThreads, 1)
+template <int D, int BLK, int MODE>
+__global__ void __launch_bounds__(AttnCfg<D>::kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap mapQ, const __grid_constant__ CUtensorMap mapK,
                 const __grid_constant__ CUtensorMap mapV, const __grid_constant__ CUtensorMap mapO,
                 const AttnParams p) {
-  using C = AttnCfg<D, BN>;
+  using C = AttnCfg<D>;
   using SS = SharedState<C::kRingK, C::kRingV>;
   static_assert(sizeof(SS) <= C::kStaticReserve, "static shared memory");
   extern __shared__ uint8_t smem_raw[];
@@ -969,15 +1018,15 @@ __global__ void __launch_bounds__(AttnCfg<D, BN>::kThreads, 1)
 
   if (warp < 8) {
     warpgroup_reg_inc<C::kRegsSoftmax>();
-    attn_softmax<D, BN, MODE>(&mapO, p, warp >> 2, tmem, out_stage, sb);
+    attn_softmax<D, BLK, MODE>(&mapO, p, warp >> 2, tmem, out_stage, sb);
   } else {
     warpgroup_reg_dec<C::kRegsOther>();
     if (warp == C::kProducerWarp) {
-      if (lane == 0) attn_producer<D, BN, MODE>(&mapQ, &mapK, &mapV, p, q_stage, ring, sb);
+      if (lane == 0) attn_producer<D, BLK, MODE>(&mapQ, &mapK, &mapV, p, q_stage, ring, sb);
     } else if (warp == C::kMmaSWarp) {
-      if (lane == 0) attn_mma_s<D, BN, MODE>(p, tmem, q_stage, ring, sb);
+      if (lane == 0) attn_mma_s<D, BLK, MODE>(p, tmem, q_stage, ring, sb);
     } else if (warp == C::kMmaPVWarp) {
-      if (lane == 0) attn_mma_pv<D, BN, MODE>(p, tmem, ring, sb);
+      if (lane == 0) attn_mma_pv<D, BLK, MODE>(p, tmem, ring, sb);
     }
   }
 
@@ -991,10 +1040,10 @@ __global__ void __launch_bounds__(AttnCfg<D, BN>::kThreads, 1)
   }
 }
 
-template <int D, int BN, int MODE>
+template <int D, int BLK, int MODE>
 cudaError_t launch_attn_instance(const AttnLaunch& L) {
-  using C = AttnCfg<D, BN>;
-  auto kern = attn_kernel<D, BN, MODE>;
+  using C = AttnCfg<D>;
+  auto kern = attn_kernel<D, BLK, MODE>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemLaunch);
   if (e != cudaSuccess) return e;
   kern<<<L.grid, C::kThreads, C::kSmemLaunch, L.stream>>>(L.mapQ, L.mapK, L.mapV, L.mapO, L.p);
@@ -1003,14 +1052,17 @@ cudaError_t launch_attn_instance(const AttnLaunch& L) {
 
 template <int D>
 cudaError_t launch_attn_for_dim(int block, int mode, const AttnLaunch& L) {
-  if (block == 128) {
-    if (mode == kDense) return launch_attn_instance<D, 128, kDense>(L);
-    if (mode == kDenseMass) return launch_attn_instance<D, 128, kDenseMass>(L);
-    return launch_attn_instance<D, 128, kSparse>(L);
+  // Plain dense attention does not depend on the block size (every sub-block
+  // is attended, causality is applied per row).
+  if (mode == kDense) return launch_attn_instance<D, 128, kDense>(L);
+  switch (block) {
+    case 128:
+      return mode == kDenseMass ? launch_attn_instance<D, 128, kDenseMass>(L) : launch_attn_instance<D, 128, kSparse>(L);
+    case 64:
+      return mode == kDenseMass ? launch_attn_instance<D, 64, kDenseMass>(L) : launch_attn_instance<D, 64, kSparse>(L);
+    default:
+      return mode == kDenseMass ? launch_attn_instance<D, 32, kDenseMass>(L) : launch_attn_instance<D, 32, kSparse>(L);
   }
-  if (mode == kDense) return launch_attn_instance<D, 64, kDense>(L);
-  if (mode == kDenseMass) return launch_attn_instance<D, 64, kDenseMass>(L);
-  return launch_attn_instance<D, 64, kSparse>(L);
 }
 
 }  // namespace wise

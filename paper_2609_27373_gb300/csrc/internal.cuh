@@ -12,13 +12,14 @@ namespace wise {
 
 enum AttnMode : int { kDense = 0, kDenseMass = 1, kSparse = 2 };
 
-// Per-CTA scratch of kDenseMass, in floats, for n_blocks key blocks:
-// log2 partial masses [2 warpgroups][2 units][n_blocks / 2 + 1 tiles][128
-// rows] (a warpgroup handles every other tile of a unit, and keeps the
-// previous unit's values until its epilogue has read them), then per-warp
-// column sums [2 warpgroups][2][4 warps][n_blocks].
-__host__ __device__ constexpr size_t scratch_floats_per_cta(int n_blocks) {
-  return (size_t)512 * (n_blocks / 2 + 1) + (size_t)16 * n_blocks;
+// Per-CTA scratch of kDenseMass, in floats, for n_tiles key tiles of 128
+// keys holding sub key blocks each (n_blocks key blocks in all): log2 partial
+// masses [2 warpgroups][2 units][n_tiles / 2 + 1][sub][128 rows] (a
+// warpgroup handles every other tile of a unit, and keeps the previous unit's
+// values until its epilogue has read them), then per-warp column sums
+// [2 warpgroups][2][4 warps][n_blocks].
+__host__ __device__ constexpr size_t scratch_floats_per_cta(int n_tiles, int sub, int n_blocks) {
+  return (size_t)512 * sub * (n_tiles / 2 + 1) + (size_t)16 * n_blocks;
 }
 
 // Bits of the per-device status word.

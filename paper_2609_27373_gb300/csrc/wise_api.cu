@@ -102,7 +102,7 @@ int check_shape(const wise_shape_t* sh, bool attention) {
       sh->head_dim <= 0 || !(sh->scale >= 0.0f) || isinf(sh->scale))
     return WISE_ERR_INVALID_ARG;
   if (sh->n_heads % sh->n_kv_heads != 0) return WISE_ERR_UNSUPPORTED;
-  if (sh->block != 64 && sh->block != 128) return WISE_ERR_UNSUPPORTED;
+  if (sh->block != 32 && sh->block != 64 && sh->block != 128) return WISE_ERR_UNSUPPORTED;
   if (attention && sh->head_dim != 64 && sh->head_dim != 96 && sh->head_dim != 128) return WISE_ERR_UNSUPPORTED;
   if (sh->seqlen % sh->block != 0) return WISE_ERR_SHAPE;
   if ((long long)sh->batch * sh->n_heads > (1LL << 24)) return WISE_ERR_UNSUPPORTED;
@@ -141,6 +141,7 @@ int launch_attention(const wise_shape_t* sh, const void* Q, const void* K, const
   }
   if (mode == kSparse) {
     if (!idx || !counts || !aligned(idx, 4) || !aligned(counts, 4) || cap <= 0) return WISE_ERR_INVALID_ARG;
+    if (cap > 65535) return WISE_ERR_UNSUPPORTED;
   }
   int err = WISE_OK;
   DeviceState* ds = device_state(&err);
@@ -150,8 +151,8 @@ int launch_attention(const wise_shape_t* sh, const void* Q, const void* K, const
   const long long outer_q = (long long)sh->batch * sh->n_heads;
   const long long outer_kv = (long long)sh->batch * sh->n_kv_heads;
   if (!make_map(&L.mapQ, Q, sh->head_dim, sh->seqlen, outer_q, 128) ||
-      !make_map(&L.mapK, K, sh->head_dim, sh->seqlen, outer_kv, sh->block) ||
-      !make_map(&L.mapV, V, sh->head_dim, sh->seqlen, outer_kv, sh->block) ||
+      !make_map(&L.mapK, K, sh->head_dim, sh->seqlen, outer_kv, 128) ||
+      !make_map(&L.mapV, V, sh->head_dim, sh->seqlen, outer_kv, 128) ||
       !make_map(&L.mapO, O, sh->head_dim, sh->seqlen, outer_q, 32))
     return WISE_ERR_CUDA;
 
@@ -179,9 +180,9 @@ int launch_attention(const wise_shape_t* sh, const void* Q, const void* K, const
   L.stream = stream;
   p.scratch = nullptr;
   if (mode == kDenseMass) {
-    // Per CTA: [nKB][2][128] log2 partial masses and [2][4][nKB] per-warp
-    // sums.
-    const size_t need = (size_t)L.grid * scratch_floats_per_cta(n_blocks) * sizeof(float);
+    // Per CTA: log2 partial masses per key sub-block and per-warp sums.
+    const size_t need =
+        (size_t)L.grid * scratch_floats_per_cta(p.n_qtiles, 128 / sh->block, n_blocks) * sizeof(float);
     if (caller_scratch) {
       if (need > caller_scratch_bytes) return WISE_ERR_UNSUPPORTED;
       p.scratch = caller_scratch;

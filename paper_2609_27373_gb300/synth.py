@@ -86,6 +86,10 @@ WORKLOADS: Dict[str, Workload] = {
                     32, 4, 0.3, 0.85, SEL_TOPK, 1, 2, 8, 0.0, 11, 3),
     "32k_gqa": Workload("32k_gqa", 1, 32768, 32, 8, 128, 128, 1.0, (5, 5), 3.0, True,
                         24, 5, 0.3, 0.85, SEL_TOPK, 1, 2, 12, 0.0, 15, 4),
+    # The 4K workload at the paper's default block of 32 keys (Sec. 5.1), with
+    # the same key budget per query block (32 blocks of 32 = 8 blocks of 128).
+    "4k_b32": Workload("4k_b32", 1, 4096, 32, 32, 128, 32, 1.0, (3, 3), 2.5, False,
+                       32, 4, 0.3, 0.85, SEL_COVERAGE, 1, 1, 0, 0.95, 32, 5),
 }
 
 

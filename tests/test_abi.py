@@ -49,7 +49,7 @@ NULL = ctypes.c_void_p(0)
 
 
 @pytest.mark.parametrize("kw,code", [
-    (dict(block=32), wise.WISE_ERR_UNSUPPORTED),
+    (dict(block=16), wise.WISE_ERR_UNSUPPORTED),
     (dict(head_dim=80), wise.WISE_ERR_UNSUPPORTED),
     (dict(n_heads=3, n_kv_heads=2), wise.WISE_ERR_UNSUPPORTED),
     (dict(seqlen=200), wise.WISE_ERR_SHAPE),

@@ -18,7 +18,7 @@ from gpu_helpers import MASS_MAX_ABS, assert_close_o, bf16_dev_to_f64, empty_lik
 pytestmark = pytest.mark.gpu
 
 
-@pytest.mark.parametrize("name", ["4k", "4k_b4_d96", "16k", "32k_gqa"])
+@pytest.mark.parametrize("name", ["4k", "4k_b4_d96", "16k", "32k_gqa", "4k_b32"])
 def test_workload_at_full_size(name):
     wl = synth.WORKLOADS[name]
     shape, sel = wise.shape_of(wl), wise.select_of(wl)

@@ -1,8 +1,9 @@
 """GPU parity of the three kernels against the fp64 oracle, through the C ABI.
 
 Sizes are small enough for the oracle to finish in seconds yet span several
-128-row query tiles, a ragged tail (a half query tile with block 64), head
-dims 64/96/128, grouped-query attention and batch > 1.
+128-row query tiles, ragged tails (a half query tile with block 64, a quarter
+or three quarters of one with block 32), head dims 64/96/128, blocks
+32/64/128, grouped-query attention and batch > 1.
 Tolerances: O within max-abs 1e-2 and rel-L2 5e-3 of fp64; per-step block
 mass within 1e-4; supports bit-exact against the oracle's selection run on
 the GPU's own fp32 masses.
@@ -25,6 +26,10 @@ CASES = {
     "d128_b64_gqa": (1, 2, 1, 384, 128, 64),
     "d96_b64": (1, 2, 2, 320, 96, 64),
     "d64_single_block": (1, 1, 1, 128, 64, 128),
+    # Block 32 (the paper's default): four query and four key blocks per tile.
+    "d128_b32": (1, 2, 2, 640, 128, 32),
+    "d64_b32_gqa_ragged": (1, 4, 2, 480, 64, 32),
+    "d96_b32_batch2": (2, 2, 1, 352, 96, 32),
 }
 
 
@@ -99,7 +104,7 @@ SELECTIONS = [
 
 
 @pytest.mark.parametrize("sel", SELECTIONS, ids=lambda s: f"m{s.mode}k{s.topk}e{s.eta}c{s.cap}s{s.n_sink}l{s.n_local}")
-@pytest.mark.parametrize("name", ["d128_b128", "d64_b64_ragged", "d128_gqa", "d96_b128_batch2"])
+@pytest.mark.parametrize("name", ["d128_b128", "d64_b64_ragged", "d128_gqa", "d96_b128_batch2", "d64_b32_gqa_ragged"])
 def test_selection_is_bit_exact(name, sel):
     shape, Q, K, V = _inputs(name, std=2.0)
     nb = shape.n_blocks
