@@ -19,7 +19,10 @@ Reported (one JSON line on rank 0):
                    pinned host memory and O copied back inside the timed region
   cpu_baseline     the fp64 oracle timed on a bounded sample on the host cores
 Multi-GPU: every rank runs an independent replica (the path has no exchange
-step); value is the max over ranks.
+step).  Times are maxima over ranks; in that time the job completes one step
+per rank, so `value` and `e2e` (ms per late step of the whole job) are the
+maximum divided by the number of ranks, while ms_per_step, dense_ms, the
+speedups and the roofline stay per replica.
 
 --impl reference times the fp64 oracle (the reference arm of this build) on
 a bounded sample of the same workload.
@@ -65,6 +68,22 @@ def sparse_traffic_bytes():
         return int(fields["traffic_bytes_per_launch"])
     except (KeyError, ValueError):
         return None
+
+
+def aggregate_over_ranks(values, world, device="cpu"):
+    """Per-rank times (ms) -> (max over ranks, whole-job time per step).
+
+    Every rank runs an independent replica, so in the slowest rank's time the
+    job completes `world` steps: the job's time per step is max / world.  With
+    world > 1 the process group must be initialised (NCCL with CUDA tensors,
+    gloo with CPU tensors)."""
+    import torch
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    mx = [float(x) for x in t.tolist()]
+    return mx, [v / world for v in mx]
 
 
 def load_peaks():
@@ -514,16 +533,14 @@ def main():
     if status != wise.WISE_OK:
         raise RuntimeError(f"kernel status: {wise.status_string(status)}")
 
-    value = statistics.mean(late_only)
     dense = statistics.mean(dense_ms)
-    per_rank = torch.tensor([value, total_ms / args.steps, e2e_ms], dtype=torch.float64, device="cuda")
-    if world > 1:
-        dist.all_reduce(per_rank, op=dist.ReduceOp.MAX)
-    value, step_ms, e2e_ms = (float(x) for x in per_rank.tolist())
+    # max over ranks; `value` and `e2e` are per late step of the whole job
+    (rank_value, step_ms, rank_e2e), (value, _, e2e_ms) = aggregate_over_ranks(
+        [statistics.mean(late_only), total_ms / args.steps, e2e_ms], world, device="cuda")
 
     peaks, peak_kind = load_peaks()
     peak = float(peaks["bf16_tflops"])
-    achieved = flops_sparse / (value * 1e-3) / 1e12
+    achieved = flops_sparse / (rank_value * 1e-3) / 1e12  # per GPU: one replica's kernel
     launches = args.steps * (wl.steps + 1)  # n_discovery dense + 1 select + n_late sparse per trajectory
 
     line = {
@@ -544,8 +561,8 @@ def main():
                    "l2": "every recurrent step has its own Q/K/V (2.9 GB rotating, > L2)",
                    "parallelism": f"replicas x{world}"},
         "dense_ms": round(dense, 5),
-        "speedup_vs_dense": round(dense / value, 4),
-        "setup_inclusive_speedup": round(n_late * dense / (statistics.mean(sel_ms) + n_late * value), 4),
+        "speedup_vs_dense": round(dense / rank_value, 4),
+        "setup_inclusive_speedup": round(n_late * dense / (statistics.mean(sel_ms) + n_late * rank_value), 4),
         "trajectory_speedup": round(wl.steps * dense / step_ms, 4),
         "discovery_ms": round(statistics.mean(disc_ms), 5),
         "select_ms": round(statistics.mean(sel_ms), 5),
