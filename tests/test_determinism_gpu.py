@@ -14,7 +14,7 @@ pytestmark = pytest.mark.gpu
 
 
 @pytest.mark.parametrize("B,H,Hkv,L,D,blk", [(1, 32, 32, 4096, 128, 128), (2, 6, 3, 2048, 96, 128),
-                                             (1, 8, 8, 1536, 64, 64)])
+                                             (1, 8, 8, 1536, 64, 64), (1, 8, 4, 2048, 128, 32)])
 def test_repeated_launches_are_bit_identical(B, H, Hkv, L, D, blk):
     shape = wise.Shape(B, L, H, Hkv, D, blk)
     nb = shape.n_blocks

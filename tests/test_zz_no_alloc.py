@@ -22,7 +22,7 @@ pytestmark = pytest.mark.gpu
 
 
 @pytest.mark.parametrize("B,H,Hkv,L,D,blk", [(1, 8, 8, 2048, 128, 128), (2, 4, 2, 1024, 64, 64),
-                                             (1, 6, 6, 768, 96, 128)])
+                                             (1, 6, 6, 768, 96, 128), (1, 4, 4, 1024, 128, 32)])
 def test_noalloc_matches_the_allocating_entry_point_on_two_calls(B, H, Hkv, L, D, blk):
     assert torch.cuda.is_available()
     shape = wise.Shape(B, L, H, Hkv, D, blk)
