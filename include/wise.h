@@ -223,6 +223,33 @@ int wise_sparse_attn(const wise_shape_t* shape, const void* Q, const void* K, co
 int wise_freeze_a_attn(const wise_shape_t* shape, const void* Q_frozen, const void* K_frozen, const void* V,
                        const int32_t* idx, const int32_t* counts, int cap, void* O, cudaStream_t stream);
 
+/* Freeze-A with a stored distribution, step 1 of 2: computes Abar of the
+ * frozen step once (definition above wise_freeze_a_attn) and stores it as
+ * Abar = P diag(inv_l).  With S = 128 / block, each 128-row query tile
+ * u = (b * n_heads + h) * ceil(seqlen / 128) + qt walks the 128-key tiles that
+ * hold blocks of its S query blocks' support lists, in ascending order; for
+ * the t-th of them, P + ((u * tile_cap + t) * 128 + row) * 128 holds the
+ * 128 x 128 bf16 tile of 2^(s - m_row) (row = query row, column = key within
+ * the tile; m_row the row's maximum logit over the support, so its largest
+ * entry is 1; exactly 0 where masked), and inv_l[u * 128 + row] = 1 / (sum of
+ * the row's entries), 0 for a row without an admissible key.
+ * P: device, n_units * tile_cap * 32 KiB, 16-byte aligned (tiles past a
+ * unit's walk are left as they are); inv_l: device fp32, n_units * 128,
+ * 4-byte aligned.  tile_cap >= min(ceil(seqlen / 128), S * cap), else
+ * WISE_ERR_INVALID_ARG.  Q_frozen, K_frozen, idx, counts and cap as in
+ * wise_sparse_attn. */
+int wise_freeze_a_probs(const wise_shape_t* shape, const void* Q_frozen, const void* K_frozen, const int32_t* idx,
+                        const int32_t* counts, int cap, void* P, float* inv_l, int tile_cap, cudaStream_t stream);
+
+/* Freeze-A with a stored distribution, step 2 of 2, once per late step:
+ *   O = Abar V = diag(inv_l) P V
+ * from P and inv_l as wise_freeze_a_probs stored them (same shape, idx,
+ * counts, cap and tile_cap) and the current step's V; a block-sparse P V
+ * product that reads the stored tiles from HBM.  O layout as in
+ * wise_sparse_attn; units without a tile give O = 0. */
+int wise_frozen_pv(const wise_shape_t* shape, const void* P, const float* inv_l, int tile_cap, const void* V,
+                   const int32_t* idx, const int32_t* counts, int cap, void* O, cudaStream_t stream);
+
 /* Overlap of two block supports A and B (e.g. the rolling working sets of two
  * consecutive steps, appendix "Stability of the Deployed Working Set"): for
  * each batch element e, over all (kv head, query block) rows,

@@ -312,24 +312,23 @@ def support_overlap(idx_a, counts_a, idx_b, counts_b):
     return out
 
 
-def freeze_a(Q0, K0, V, idx, counts, block, scale=None):
-    """Freeze-A control (appendix "Experimental details", intervention
-    controls), in the order the paper defines it: A = the unrestricted causal
-    attention of the frozen step (softmax of scale * Q0 K0^T + M, Eq. 2),
-    Abar = A restricted to the key blocks of the support and renormalised over
-    the admissible keys, O = Abar V with the current step's V.  fp64 numpy.
-    Q0 [B,H,L,d], K0 and V [B,Hkv,L,d] (any float dtype), idx [B,Hkv,nQB,cap],
-    counts [B,Hkv,nQB].  Rows whose restricted mass is zero give O = 0."""
+def freeze_a_distribution(Q0, K0, idx, counts, block, scale=None):
+    """Abar of the Freeze-A control (appendix "Experimental details",
+    intervention controls), in the order the paper defines it: A = the
+    unrestricted causal attention of the frozen step (softmax of
+    scale * Q0 K0^T + M, Eq. 2), then A restricted to the key blocks of the
+    support and renormalised over the admissible keys.  fp64 numpy, [B,H,L,L];
+    rows whose restricted mass is zero are 0.  Q0 [B,H,L,d], K0 [B,Hkv,L,d],
+    idx [B,Hkv,nQB,cap], counts [B,Hkv,nQB]."""
     Q0 = np.asarray(Q0, dtype=np.float64)
     K0 = np.asarray(K0, dtype=np.float64)
-    V = np.asarray(V, dtype=np.float64)
     B, H, L, d = Q0.shape
     Hkv = K0.shape[1]
     group = H // Hkv
     sc = 1.0 / np.sqrt(d) if scale is None else float(scale)
     nq = L // block
     causal = np.tril(np.ones((L, L), dtype=bool))
-    out = np.zeros((B, H, L, V.shape[3]), dtype=np.float64)
+    out = np.zeros((B, H, L, L), dtype=np.float64)
     for b in range(B):
         for h in range(H):
             g = h // group
@@ -343,6 +342,19 @@ def freeze_a(Q0, K0, V, idx, counts, block, scale=None):
                     keep[q * block:(q + 1) * block, v * block:(v + 1) * block] = True
             abar = np.where(keep & causal, a, 0.0)
             tot = abar.sum(axis=1, keepdims=True)
-            abar = np.divide(abar, tot, out=np.zeros_like(abar), where=tot > 0)
-            out[b, h] = abar @ V[b, g]
+            out[b, h] = np.divide(abar, tot, out=np.zeros_like(abar), where=tot > 0)
+    return out
+
+
+def freeze_a(Q0, K0, V, idx, counts, block, scale=None):
+    """Freeze-A output O = Abar V with the current step's V [B,Hkv,L,dv]
+    (Abar from freeze_a_distribution).  fp64, [B,H,L,dv]."""
+    abar = freeze_a_distribution(Q0, K0, idx, counts, block, scale)
+    V = np.asarray(V, dtype=np.float64)
+    B, H = abar.shape[:2]
+    group = H // V.shape[1]
+    out = np.zeros((B, H, abar.shape[2], V.shape[3]), dtype=np.float64)
+    for b in range(B):
+        for h in range(H):
+            out[b, h] = abar[b, h] @ V[b, h // group]
     return out

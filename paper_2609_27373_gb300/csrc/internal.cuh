@@ -103,6 +103,24 @@ struct SupportMassParams {
   int* status;
 };
 
+// Freeze-A with a stored distribution (freeze.cu).  For unit u (the 128-row
+// query tile qt of (b, h), u = (b * n_heads + h) * n_qtiles + qt) and the
+// t-th key tile of its support walk, P + ((u * tile_cap + t) * 128 + row) * 128
+// holds the bf16 tile of 2^(s - m_row); inv_l[u * 128 + row] = 1 / (row sum),
+// so that Abar = diag(inv_l) P.
+struct FreezeLaunch {
+  CUtensorMap mapQ, mapK;  // wise_freeze_a_probs: the frozen step's Q and K (128-row boxes)
+  CUtensorMap mapV, mapP;  // wise_frozen_pv: current V, and P viewed as [tiles][128][128]
+  AttnParams p;            // shape, support lists, scale, status; O for wise_frozen_pv
+  __nv_bfloat16* P;
+  float* inv_l;
+  int tile_cap;
+  int grid;  // wise_frozen_pv: persistent grid, min(n_units, SM count)
+  cudaStream_t stream;
+};
+cudaError_t launch_freeze_probs(int head_dim, int block, const FreezeLaunch& L);
+cudaError_t launch_frozen_pv(int head_dim, int block, const FreezeLaunch& L);
+
 struct SupportOverlapParams {
   int batch, rows;  // rows per batch element: n_kv_heads * n_blocks
   int n_blocks, cap_a, cap_b;

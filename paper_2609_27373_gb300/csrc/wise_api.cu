@@ -1,6 +1,9 @@
 // Host side of the C ABI declared in include/wise.h: argument checks, TMA
 // tensor maps, the per-device scratch buffer and status word, and launches.
 #include <limits.h>
+#include <string.h>
+
+#include <algorithm>
 #include <math.h>
 #include <mutex>
 
@@ -222,6 +225,85 @@ extern "C" int wise_freeze_a_attn(const wise_shape_t* shape, const void* Q_froze
   // softmax over the support of the frozen step's logits, so the sparse kernel
   // computes it from that step's Q and K against the current V.
   return launch_attention(shape, Q_frozen, K_frozen, V, O, kSparse, nullptr, 0, idx, counts, cap, stream);
+}
+
+namespace {
+
+// Shared checks and parameters of the two stored-distribution calls.
+int freeze_setup(const wise_shape_t* sh, const int32_t* idx, const int32_t* counts, int cap, const void* P,
+                 const float* inv_l, int tile_cap, FreezeLaunch& L) {
+  int rc = check_shape(sh, true);
+  if (rc != WISE_OK) return rc;
+  if (cap <= 0 || !P || !aligned(P, 16) || !inv_l || !aligned(inv_l, 4)) return WISE_ERR_INVALID_ARG;
+  if (cap > 65535) return WISE_ERR_UNSUPPORTED;
+  if (sh->batch == 0 || sh->seqlen == 0) return WISE_OK;
+  if (!idx || !counts || !aligned(idx, 4) || !aligned(counts, 4)) return WISE_ERR_INVALID_ARG;
+  const int n_qtiles = (sh->seqlen + 127) / 128;
+  const long long walk_max = std::min<long long>(n_qtiles, (long long)(128 / sh->block) * cap);
+  if (tile_cap < walk_max) return WISE_ERR_INVALID_ARG;
+  const long long units = (long long)sh->batch * sh->n_heads * n_qtiles;
+  if (units * tile_cap > INT32_MAX) return WISE_ERR_UNSUPPORTED;
+  int err = WISE_OK;
+  DeviceState* ds = device_state(&err);
+  if (!ds) return err;
+  AttnParams& p = L.p;
+  memset(&p, 0, sizeof(p));
+  p.batch = sh->batch;
+  p.seqlen = sh->seqlen;
+  p.n_heads = sh->n_heads;
+  p.n_kv_heads = sh->n_kv_heads;
+  p.group = sh->n_heads / sh->n_kv_heads;
+  p.n_qtiles = n_qtiles;
+  p.n_blocks = sh->seqlen / sh->block;
+  p.n_units = (int)units;
+  const float scale = sh->scale > 0.0f ? sh->scale : 1.0f / sqrtf((float)sh->head_dim);
+  p.scale_log2 = scale * 1.4426950408889634f;
+  p.idx = idx;
+  p.counts = counts;
+  p.cap = cap;
+  p.status = ds->status;
+  L.P = reinterpret_cast<__nv_bfloat16*>(const_cast<void*>(P));
+  L.inv_l = const_cast<float*>(inv_l);
+  L.tile_cap = tile_cap;
+  return WISE_OK;
+}
+
+}  // namespace
+
+extern "C" int wise_freeze_a_probs(const wise_shape_t* shape, const void* Q_frozen, const void* K_frozen,
+                                   const int32_t* idx, const int32_t* counts, int cap, void* P, float* inv_l,
+                                   int tile_cap, cudaStream_t stream) {
+  FreezeLaunch L;
+  int rc = freeze_setup(shape, idx, counts, cap, P, inv_l, tile_cap, L);
+  if (rc != WISE_OK || shape->batch == 0 || shape->seqlen == 0) return rc;
+  if (!Q_frozen || !K_frozen || !aligned(Q_frozen, 16) || !aligned(K_frozen, 16)) return WISE_ERR_INVALID_ARG;
+  const long long outer_q = (long long)shape->batch * shape->n_heads;
+  const long long outer_kv = (long long)shape->batch * shape->n_kv_heads;
+  if (!make_map(&L.mapQ, Q_frozen, shape->head_dim, shape->seqlen, outer_q, 128) ||
+      !make_map(&L.mapK, K_frozen, shape->head_dim, shape->seqlen, outer_kv, 128))
+    return WISE_ERR_CUDA;
+  L.stream = stream;
+  return launch_freeze_probs(shape->head_dim, shape->block, L) == cudaSuccess ? WISE_OK : WISE_ERR_CUDA;
+}
+
+extern "C" int wise_frozen_pv(const wise_shape_t* shape, const void* P, const float* inv_l, int tile_cap,
+                              const void* V, const int32_t* idx, const int32_t* counts, int cap, void* O,
+                              cudaStream_t stream) {
+  FreezeLaunch L;
+  int rc = freeze_setup(shape, idx, counts, cap, P, inv_l, tile_cap, L);
+  if (rc != WISE_OK || shape->batch == 0 || shape->seqlen == 0) return rc;
+  if (!V || !O || !aligned(V, 16) || !aligned(O, 16)) return WISE_ERR_INVALID_ARG;
+  const long long outer_kv = (long long)shape->batch * shape->n_kv_heads;
+  if (!make_map(&L.mapV, V, shape->head_dim, shape->seqlen, outer_kv, 128) ||
+      !make_map(&L.mapP, P, 128, 128, (long long)L.p.n_units * tile_cap, 128))
+    return WISE_ERR_CUDA;
+  L.p.O = reinterpret_cast<__nv_bfloat16*>(O);
+  int err = WISE_OK;
+  DeviceState* ds = device_state(&err);
+  if (!ds) return err;
+  L.grid = L.p.n_units < ds->sm_count ? L.p.n_units : ds->sm_count;
+  L.stream = stream;
+  return launch_frozen_pv(shape->head_dim, shape->block, L) == cudaSuccess ? WISE_OK : WISE_ERR_CUDA;
 }
 
 extern "C" int wise_select_support(const wise_shape_t* shape, const wise_select_t* sel, const float* blockmass,

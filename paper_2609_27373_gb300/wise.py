@@ -27,7 +27,8 @@ WISE_SEL_TOPK = 0
 WISE_SEL_COVERAGE = 1
 
 EXPORTS = ("wise_full_attn_accumulate", "wise_full_attn_accumulate_noalloc", "wise_select_support",
-           "wise_sparse_attn", "wise_freeze_a_attn", "wise_support_mass", "wise_support_overlap",
+           "wise_sparse_attn", "wise_freeze_a_attn", "wise_freeze_a_probs", "wise_frozen_pv", "wise_support_mass",
+           "wise_support_overlap",
            "wise_select_working_set", "wise_get_status", "wise_status_string", "wise_version")
 NOALLOC_SCRATCH_BYTES = 8 << 20
 
@@ -103,6 +104,9 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.wise_select_support.argtypes = [ctypes.POINTER(wise_shape_t), ctypes.POINTER(wise_select_t), P, P, P, P]
         lib.wise_sparse_attn.argtypes = [ctypes.POINTER(wise_shape_t), P, P, P, P, P, ctypes.c_int, P, P]
         lib.wise_freeze_a_attn.argtypes = [ctypes.POINTER(wise_shape_t), P, P, P, P, P, ctypes.c_int, P, P]
+        lib.wise_freeze_a_probs.argtypes = [ctypes.POINTER(wise_shape_t), P, P, P, P, ctypes.c_int, P, P,
+                                            ctypes.c_int, P]
+        lib.wise_frozen_pv.argtypes = [ctypes.POINTER(wise_shape_t), P, P, ctypes.c_int, P, P, P, ctypes.c_int, P, P]
         lib.wise_support_mass.argtypes = [ctypes.POINTER(wise_shape_t), P, P, P, ctypes.c_int, P, P]
         I = ctypes.c_int
         lib.wise_support_overlap.argtypes = [ctypes.POINTER(wise_shape_t), P, P, I, P, P, I, P, P]
@@ -228,6 +232,57 @@ def wise_freeze_a_attn(shape: Shape, Q_frozen, K_frozen, V, idx, counts, O, stre
                                    _ptr(counts), int(cap), _ptr(O), _stream(stream))
     if rc != WISE_OK:
         raise WiseError(rc, "wise_freeze_a_attn")
+
+
+def freeze_tile_cap(shape: Shape, cap: int) -> int:
+    """Smallest tile_cap the stored-distribution calls accept for support
+    lists of row width `cap`."""
+    return min((shape.seqlen + 127) // 128, (128 // shape.block) * cap)
+
+
+def wise_freeze_a_probs(shape: Shape, Q_frozen, K_frozen, idx, counts, P, inv_l, stream=None) -> None:
+    """Stores Abar of the frozen step as P bf16 [n_units, tile_cap, 128, 128]
+    (row-max-relative exponentials) and inv_l fp32 [n_units, 128]."""
+    _check(Q_frozen, "Q_frozen", (shape.batch, shape.n_heads, shape.seqlen, shape.head_dim), torch.bfloat16)
+    _check(K_frozen, "K_frozen", (shape.batch, shape.n_kv_heads, shape.seqlen, shape.head_dim), torch.bfloat16)
+    cap = _support(shape, idx, counts)
+    tile_cap = _p_tiles(shape, P, inv_l)
+    sh = shape.c()
+    rc = load().wise_freeze_a_probs(ctypes.byref(sh), _ptr(Q_frozen), _ptr(K_frozen), _ptr(idx), _ptr(counts), cap,
+                                    _ptr(P), _ptr(inv_l), tile_cap, _stream(stream))
+    if rc != WISE_OK:
+        raise WiseError(rc, "wise_freeze_a_probs")
+
+
+def wise_frozen_pv(shape: Shape, P, inv_l, V, idx, counts, O, stream=None) -> None:
+    """O = Abar V from the P and inv_l that wise_freeze_a_probs stored."""
+    _check(V, "V", (shape.batch, shape.n_kv_heads, shape.seqlen, shape.head_dim), torch.bfloat16)
+    _check(O, "O", (shape.batch, shape.n_heads, shape.seqlen, shape.head_dim), torch.bfloat16)
+    cap = _support(shape, idx, counts)
+    tile_cap = _p_tiles(shape, P, inv_l)
+    sh = shape.c()
+    rc = load().wise_frozen_pv(ctypes.byref(sh), _ptr(P), _ptr(inv_l), tile_cap, _ptr(V), _ptr(idx), _ptr(counts),
+                               cap, _ptr(O), _stream(stream))
+    if rc != WISE_OK:
+        raise WiseError(rc, "wise_frozen_pv")
+
+
+def _support(shape: Shape, idx, counts) -> int:
+    if idx is None or idx.dim() != 4:
+        raise ValueError("idx must be int32 [batch, n_kv_heads, nQB, cap]")
+    cap = int(idx.shape[3])
+    _check(idx, "idx", (shape.batch, shape.n_kv_heads, shape.n_blocks, cap), torch.int32)
+    _check(counts, "counts", (shape.batch, shape.n_kv_heads, shape.n_blocks), torch.int32)
+    return cap
+
+
+def _p_tiles(shape: Shape, P, inv_l) -> int:
+    n_units = shape.batch * shape.n_heads * ((shape.seqlen + 127) // 128)
+    if P is None or P.dim() != 4:
+        raise ValueError("P must be bf16 [n_units, tile_cap, 128, 128]")
+    _check(P, "P", (n_units, int(P.shape[1]), 128, 128), torch.bfloat16)
+    _check(inv_l, "inv_l", (n_units, 128), torch.float32)
+    return int(P.shape[1])
 
 
 def wise_support_overlap(shape: Shape, idx_a, counts_a, idx_b, counts_b, inter_union, stream=None) -> None:

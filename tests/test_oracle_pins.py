@@ -607,3 +607,21 @@ def test_freeze_a_rows_are_convex_combinations_of_supported_values():
     got = np.stack(got_rows)
     np.testing.assert_allclose(got[..., 0], 1.0, rtol=0, atol=1e-12)
     np.testing.assert_allclose(got[..., 1], 0.0, rtol=0, atol=1e-12)
+
+
+def test_freeze_a_distribution_rows_are_normalised_on_the_support():
+    """Abar is a distribution over the admissible supported keys of each row
+    (rows of a query block with an empty list are 0), zero elsewhere."""
+    B, H, Hkv, L, D, blk = 1, 2, 1, 48, 4, 8
+    Q, K, _ = synth.random_qkv(B, H, Hkv, L, D, seed=27)
+    idx, counts = synth.random_support(B, Hkv, L // blk, 3, seed=28)
+    counts[0, 0, 2] = 0
+    abar = orc.freeze_a_distribution(bf16_vals(Q), bf16_vals(K), idx, counts, blk)
+    for h in range(H):
+        for i in range(L):
+            q = i // blk
+            sup = set(int(v) for v in idx[0, 0, q, :counts[0, 0, q]])
+            allowed = np.array([(j // blk in sup) and j <= i for j in range(L)])
+            assert np.all(abar[0, h, i, ~allowed] == 0.0)
+            want = 1.0 if allowed.any() else 0.0
+            assert abs(abar[0, h, i].sum() - want) < 1e-12
