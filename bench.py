@@ -226,8 +226,9 @@ def run_reference(args):
 
 def run_profile_sequence():
     """Fixed launch sequence for profilers: n_discovery dense+mass launches,
-    one selection, two sparse launches and one plain dense launch of the 4K
-    workload (about 0.7 GB on the device)."""
+    one selection, two sparse launches, one plain dense launch, one Freeze-A
+    store and two stored-Freeze-A P V launches of the 4K workload (about 1 GB
+    on the device)."""
     import torch
     from paper_2609_27373_gb300 import synth, wise
     wl = synth.WORKLOADS[WORKLOAD]
@@ -240,6 +241,13 @@ def run_profile_sequence():
         layer.step(t, Q, K, V, O)
     wise.wise_sparse_attn(shape, Q, K, V, layer.idx, layer.counts, O)
     wise.wise_full_attn_accumulate(shape, Q, K, V, O)
+    # Freeze-A with the distribution stored once, then two late-step P V launches
+    n_units = wl.batch * wl.n_heads * (wl.seqlen // 128)
+    P = torch.empty((n_units, wise.freeze_tile_cap(shape, wl.cap), 128, 128), dtype=torch.bfloat16, device="cuda")
+    inv_l = torch.empty((n_units, 128), dtype=torch.float32, device="cuda")
+    wise.wise_freeze_a_probs(shape, Q, K, layer.idx, layer.counts, P, inv_l)
+    for _ in range(2):
+        wise.wise_frozen_pv(shape, P, inv_l, V, layer.idx, layer.counts, O)
     status = wise.wise_get_status()
     if status != wise.WISE_OK:
         raise RuntimeError(wise.status_string(status))
