@@ -576,6 +576,39 @@ def main():
                "tile_density": round(tiles32 / causal_tiles, 4), "speedup_vs_dense": round(statistics.mean(dense_ms) / b32_ms, 4)}
     del steps32, layer32, O32
 
+    # ---- the other benchmark workloads at their full sizes: own discovery
+    # and selection, then late steps timed against the dense kernel on the
+    # same inputs (context for the 4K line; parity is tested separately)
+    other = {}
+    for name in ("tiny", "4k_b4_d96", "16k", "32k_gqa"):
+        wo = synth.WORKLOADS[name]
+        sh_o, sel_o = wise.shape_of(wo), wise.select_of(wo)
+        lay_o = wise.WiseAttention(sh_o, sel_o, wo.n_discovery)
+        tr_o = synth.Trajectory(wo)
+        n_t = 4
+        st_o = [tuple(torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).cuda() for x in tr_o.step(t))
+                for t in range(wo.n_discovery + n_t)]
+        O_o = torch.empty_like(st_o[0][0])
+        for t in range(wo.n_discovery + 1):
+            lay_o.step(t, *st_o[t], O_o)
+        ev_o = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(2 * n_t)]
+        for rep in range(2):  # the first pass warms up
+            for i, t in enumerate(range(wo.n_discovery, wo.n_discovery + n_t)):
+                ev_o[i][0].record(stream)
+                wise.wise_sparse_attn(sh_o, *st_o[t], lay_o.idx, lay_o.counts, O_o)
+                ev_o[i][1].record(stream)
+                ev_o[n_t + i][0].record(stream)
+                wise.wise_full_attn_accumulate(sh_o, *st_o[t], O_o)
+                ev_o[n_t + i][1].record(stream)
+            torch.cuda.synchronize()
+        sp = statistics.mean(a.elapsed_time(b) for a, b in ev_o[:n_t])
+        dn = statistics.mean(a.elapsed_time(b) for a, b in ev_o[n_t:])
+        f_o = sparse_flops(lay_o.idx.cpu().numpy(), lay_o.counts.cpu().numpy(), wo.n_heads, wo.head_dim, wo.block)
+        other[name] = {"late_ms": round(sp, 5), "dense_ms": round(dn, 5), "speedup_vs_dense": round(dn / sp, 4),
+                       "tflops_effective": round(f_o / (sp * 1e-3) / 1e12, 2),
+                       "density": round(f_o / dense_flops(wo.batch, wo.n_heads, wo.seqlen, wo.head_dim), 4)}
+        del st_o, lay_o, O_o
+
     # ---- the whole trajectory as one CUDA graph (discovery, selection, late
     # steps), replayed; its launches carry no host-side gaps
     graph = {"ms": None, "note": None}
@@ -645,6 +678,7 @@ def main():
         "supports": supports,
         "rolling_jaccard_at_discovery_end": round(rolling_jaccard, 4),
         "block32": block32,
+        "other_workloads": other,
         "freeze_a_ms": round(freeze_a_ms, 5),
         "freeze_a_stored": frozen,
         "all_blocks_vs_dense": round(all_blocks_ms / dense, 4),
