@@ -117,8 +117,8 @@ struct AttnCfg {
   // completes warpgroup 2 for setmaxnreg).  Launch: 384 x 168 registers;
   // after the split 256 x kRegsSoftmax + 128 x kRegsOther = 64512.
   static constexpr int kThreads = 384;
-  static constexpr int kRegsSoftmax = 224;
-  static constexpr int kRegsOther = 56;
+  static constexpr int kRegsSoftmax = 216;
+  static constexpr int kRegsOther = 72;
   static constexpr int kProducerWarp = 8;
   static constexpr int kMmaSWarp = 9;   // issues S = Q K^T, owns the TMEM allocation
   static constexpr int kMmaPVWarp = 10; // issues O += P V
