@@ -148,7 +148,7 @@ __global__ void __launch_bounds__(160, 1)
         }
         tc_fence_after_sync();
         const uint64_t b0 = smem_desc_sw128(smem_u32(ring + slot * C::kKBytes), 16, 1024);
-#pragma unroll 1
+#pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t a_off = ((kk >> 2) * (128 * 128) + (kk & 3) * 32) >> 4;
           const uint32_t b_off = ((kk >> 2) * (kTileN * 128) + (kk & 3) * 32) >> 4;
@@ -340,7 +340,7 @@ __global__ void __launch_bounds__(192, 1)
           const uint32_t st = smem_u32(ring + slot * kStage);
           const uint64_t a0 = smem_desc_sw128(st, 16, 1024);
           const uint64_t b0 = smem_desc_sw128(st + C::kPBytes, kTileN * 128, 1024);
-#pragma unroll 1
+#pragma unroll
           for (int kk = 0; kk < kTileN / 16; ++kk) {
             const uint32_t a_off = ((kk >> 2) * (128 * 128) + (kk & 3) * 32) >> 4;
             umma_bf16_ss(tmem + ob * 128, a0 + a_off, b0 + ((kk * 2048) >> 4), idesc, (t > 0 || kk > 0) ? 1u : 0u);
