@@ -127,11 +127,9 @@ struct AttnCfg {
   static_assert(256 * kRegsSoftmax + 128 * kRegsOther <= kThreads * 168, "register split");
 };
 
-// Tile schedule rings.  Entry = {key tile | mask << 16, batch * n_heads +
-// head, flags, tile index within its unit | query tile << 16} (for the end
-// marker: {0, 0, kEntEnd, number of tiles}); carrying the unit's coordinates
-// spares the softmax warps the integer divisions of decoding a unit index.
-// With S = 128 / block query blocks per query tile and key blocks
+// Tile schedule rings.  Entry = {key tile | mask << 16, unit, flags, tile
+// index within its unit} (for the end marker: {0, 0, kEntEnd, number of
+// tiles}).  With S = 128 / block query blocks per query tile and key blocks
 // per key tile, bit qi * S + ki of the mask says that query block qi of the
 // tile attends key block ki of the key tile.  Flag bits 8 and up hold the
 // index of the unit among this CTA's units with tiles.
@@ -381,13 +379,13 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
   // Writes the next entry of a ring.  Its position follows from the counts:
   // the MMA ring holds every tile, ring 1 the odd tiles, ring 0 the even
   // tiles and the units without tiles.
-  auto emit = [&](int ring_w, int kb, int bh, int flags, int t) -> bool {
+  auto emit = [&](int ring_w, int kb, int u, int flags, int t) -> bool {
     const int e = ring_w == kMmaRing ? jt : ring_w == 1 ? (jt >> 1) : ((jt + 1) >> 1) + n_empty;
     const int slot = e % kSchedSlots;
     if (e >= kSchedSlots &&
         !mbar_wait(&sb.sched_empty[ring_w][slot], ((e / kSchedSlots) - 1) & 1, abort))
       return false;
-    sb.sched[ring_w][slot] = make_int4(kb, bh, flags, t);
+    sb.sched[ring_w][slot] = make_int4(kb, u, flags, t);
     mbar_arrive(&sb.sched_full[ring_w][slot]);  // release: the entry is visible to whoever acquires the phase
     return true;
   };
@@ -416,7 +414,7 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
     uint32_t mask;
     bool have = it.next(kb, mask);
     if (!have) {
-      if (!emit(0, 0, b * p.n_heads + h, kEntEmpty, qt << 16)) ok = false;
+      if (!emit(0, 0, u, kEntEmpty, 0)) ok = false;
       ++n_empty;
     }
     bool first = true;
@@ -427,8 +425,7 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
       const bool more = it.next(nkb, nmask);
       const int flags = (first ? kEntFirst : 0) | (more ? 0 : kEntLast) | (unit_ix << kEntUnitShift);
       const int key = (int)((uint32_t)kb | (mask << 16));
-      const int tq = t | (qt << 16);
-      if (!emit(kMmaRing, key, b * p.n_heads + h, flags, tq) || !emit(jt & 1, key, b * p.n_heads + h, flags, tq)) {
+      if (!emit(kMmaRing, key, u, flags, t) || !emit(jt & 1, key, u, flags, t)) {
         ok = false;
         break;
       }
@@ -536,7 +533,7 @@ __device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* q_stage,
     tc_fence_after_sync();
     const uint32_t s_col = C::kTmemS;
     const uint64_t b0 = smem_desc_sw128(smem_u32(ring + slot * C::kKVBytes), 16, 1024);
-#pragma unroll
+#pragma unroll 1
     for (int kk = 0; kk < D / 16; ++kk) {
       // K step kk: 8 TMEM columns of Q; shared-memory descriptors of later
       // steps differ only in the start address field (address >> 4).
@@ -651,8 +648,7 @@ __device__ __forceinline__ void load_s_row(uint32_t addr, float (&s)[kTileN], ui
 
 // What the epilogue needs about its unit.
 struct EpiInfo {
-  int bh;     // batch * n_heads + head of the unit
-  int qt;     // its query tile
+  int u;      // unit
   int j0;     // tile counter of its first tile
   int j1;     // tile counter of its last tile
   int nu;     // index among this CTA's units with tiles
@@ -803,7 +799,8 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     tc_fence_before_sync();
     __syncwarp();
     if (lane == 0) mbar_arrive(&sb.o_free);
-    const int bh = ei.bh, qt = ei.qt;
+    int b, h, qt;
+    decode_unit(p, ei.u, b, h, qt);
     const int row = qt * 128 + r;
     const float inv_l = l_row > 0.0f ? 1.0f / l_row : 0.0f;
     // O / l through this warp's staging box (32 rows x 64 columns, 128-byte
@@ -828,7 +825,7 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) {
-        tma_store_3d(mapO, stage, hb * 64, qt * 128 + wq * 32, bh);
+        tma_store_3d(mapO, stage, hb * 64, qt * 128 + wq * 32, b * p.n_heads + h);
         tma_store_commit();
       }
     }
@@ -859,7 +856,7 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
         const int qi = e / p.n_blocks, kb = e % p.n_blocks;
         const int qblock = qt * S + qi;
         if (qblock >= p.n_blocks) continue;
-        float* out = p.blockmass + ((size_t)bh * p.n_blocks + qblock) * p.n_blocks + kb;
+        float* out = p.blockmass + ((size_t)(b * p.n_heads + h) * p.n_blocks + qblock) * p.n_blocks + kb;
         if (kb < n_kb) {
           float sum = 0.0f;
 #pragma unroll
@@ -914,9 +911,11 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     if (fl & kEntEmpty) {
       // No key tile (ring 0 only): the rows of the unit attend nothing and
       // are zero.
-      const int row = (ent.w >> 16) * 128 + r;
+      int b, h, qt;
+      decode_unit(p, ent.y, b, h, qt);
+      const int row = qt * 128 + r;
       if (row < p.seqlen) {
-        uint4* dst = reinterpret_cast<uint4*>(p.O + ((size_t)ent.y * p.seqlen + row) * D);
+        uint4* dst = reinterpret_cast<uint4*>(p.O + ((size_t)(b * p.n_heads + h) * p.seqlen + row) * D);
 #pragma unroll
         for (int c = 0; c < D / 8; ++c) dst[c] = make_uint4(0u, 0u, 0u, 0u);
       }
@@ -930,19 +929,20 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
       break;
     }
     if (fresh) {
-      cur_row = (ent.w >> 16) * 128 + r;
+      int b, h, qt;
+      decode_unit(p, ent.y, b, h, qt);
+      cur_row = qt * 128 + r;
       l_w = 0.0f;
       m_w = -INFINITY;
     }
-    const int t = ent.w & 0xFFFF;
-    if (!tile(ent.x, first, t, fl >> kEntUnitShift)) {
+    if (!tile(ent.x, first, ent.w, fl >> kEntUnitShift)) {
       ok = false;
       break;
     }
     fresh = false;
     if (fl & kEntLast) {
       // L: this warpgroup handled the unit's last tile.
-      const EpiInfo ei{ent.y, ent.w >> 16, j - t, j, fl >> kEntUnitShift, (ent.x & 0xFFFF) + 1, l_w, m_w};
+      const EpiInfo ei{ent.y, j - ent.w, j, fl >> kEntUnitShift, (ent.x & 0xFFFF) + 1, l_w, m_w};
       if (!epilogue(ei)) {
         ok = false;
         break;
