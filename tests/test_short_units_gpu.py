@@ -1,0 +1,58 @@
+"""Full-size sparse steps whose units are one or two key tiles long.
+
+With such supports a unit ends at nearly every tile, so the warpgroup that
+handled a unit's last tile writes O out while the other starts the next
+unit, tile after tile.  The two warpgroups share the output staging boxes;
+a missing order between one warpgroup's TMA stores reading a box and the
+other's next writes into it would show up here as wrong or unrepeatable
+rows.  Every row is checked against the oracle, and repeated launches must
+agree bit for bit.  V is drawn with std 0.5: a row that attends only the
+first few keys of its diagonal block is close to one V row, and at the
+std-1 tail (|V| ~ 5) half a bf16 ulp of the output alone is 0.016, above the
+1e-2 bound; below 4 it is at most 0.008.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as orc
+from paper_2609_27373_gb300 import synth, wise
+from gpu_helpers import assert_close_o, bf16_dev_to_f64, empty_like_q, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+def short_support(n_kv_heads, n_blocks, pattern):
+    """Query block q attends block q alone ("diagonal"), or the sink block 0
+    and block q for every third q ("diagonal_or_sink"); ascending, -1 padded."""
+    idx = np.full((1, n_kv_heads, n_blocks, 2), -1, dtype=np.int32)
+    counts = np.ones((1, n_kv_heads, n_blocks), dtype=np.int32)
+    for q in range(n_blocks):
+        if pattern == "diagonal_or_sink" and q > 0 and q % 3 == 1:
+            idx[0, :, q, :2] = (0, q)
+            counts[0, :, q] = 2
+        else:
+            idx[0, :, q, 0] = q
+    return idx, counts
+
+
+@pytest.mark.parametrize("blk", [128, 32])
+@pytest.mark.parametrize("pattern", ["diagonal", "diagonal_or_sink"])
+def test_one_and_two_tile_units_at_4k(blk, pattern):
+    B, H, L, D = 1, 32, 4096, 128
+    shape = wise.Shape(B, L, H, H, D, blk)
+    Q, K, V = synth.random_qkv(B, H, H, L, D, seed=17, std=1.3, v_std=0.5)
+    dq, dk, dv = to_dev(Q), to_dev(K), to_dev(V)
+    idx, counts = short_support(H, shape.n_blocks, pattern)
+    di, dc = torch.from_numpy(idx).cuda(), torch.from_numpy(counts).cuda()
+    outs = []
+    for _ in range(4):
+        O = empty_like_q(Q)
+        wise.wise_sparse_attn(shape, dq, dk, dv, di, dc, O)
+        outs.append(O)
+    torch.cuda.synchronize()
+    assert wise.wise_get_status() == wise.WISE_OK
+    for O in outs[1:]:
+        assert torch.equal(O.view(torch.int16), outs[0].view(torch.int16)), "repeated launches differ"
+    want = orc.sparse_attention(Q, K, V, idx, counts, blk)
+    assert_close_o(bf16_dev_to_f64(outs[0]), want, what=f"{pattern} block {blk}")
