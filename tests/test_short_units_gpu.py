@@ -36,14 +36,18 @@ def short_support(n_kv_heads, n_blocks, pattern):
     return idx, counts
 
 
-@pytest.mark.parametrize("blk", [128, 32])
-@pytest.mark.parametrize("pattern", ["diagonal", "diagonal_or_sink"])
-def test_one_and_two_tile_units_at_4k(blk, pattern):
-    B, H, L, D = 1, 32, 4096, 128
-    shape = wise.Shape(B, L, H, H, D, blk)
-    Q, K, V = synth.random_qkv(B, H, H, L, D, seed=17, std=1.3, v_std=0.5)
+@pytest.mark.parametrize("D,Hkv,blk,pattern", [
+    (128, 32, 128, "diagonal"), (128, 32, 128, "diagonal_or_sink"),
+    (128, 32, 32, "diagonal"), (128, 32, 32, "diagonal_or_sink"),
+    (96, 32, 128, "diagonal_or_sink"),   # two staging boxes, the second half empty
+    (64, 8, 64, "diagonal_or_sink"),     # one staging box; four query heads per kv head
+])
+def test_one_and_two_tile_units_at_4k(D, Hkv, blk, pattern):
+    B, H, L = 1, 32, 4096
+    shape = wise.Shape(B, L, H, Hkv, D, blk)
+    Q, K, V = synth.random_qkv(B, H, Hkv, L, D, seed=17, std=1.3, v_std=0.5)
     dq, dk, dv = to_dev(Q), to_dev(K), to_dev(V)
-    idx, counts = short_support(H, shape.n_blocks, pattern)
+    idx, counts = short_support(Hkv, shape.n_blocks, pattern)
     di, dc = torch.from_numpy(idx).cuda(), torch.from_numpy(counts).cuda()
     outs = []
     for _ in range(4):
@@ -55,4 +59,4 @@ def test_one_and_two_tile_units_at_4k(blk, pattern):
     for O in outs[1:]:
         assert torch.equal(O.view(torch.int16), outs[0].view(torch.int16)), "repeated launches differ"
     want = orc.sparse_attention(Q, K, V, idx, counts, blk)
-    assert_close_o(bf16_dev_to_f64(outs[0]), want, what=f"{pattern} block {blk}")
+    assert_close_o(bf16_dev_to_f64(outs[0]), want, what=f"{pattern} d {D} kv heads {Hkv} block {blk}")
