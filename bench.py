@@ -35,6 +35,7 @@ import os
 import statistics
 import subprocess
 import sys
+import tempfile
 import time
 
 import numpy as np
@@ -261,6 +262,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--clocks-dir", default=None,
+                    help="directory for the nvidia-smi clock samples of the timed region (default: the temp dir)")
     ap.add_argument("--profile", action="store_true",
                     help="no timing: the 4K discovery steps, one selection, then 2 late sparse and 1 dense launches "
                          "(a small, fixed launch sequence for ncu captures)")
@@ -320,8 +323,7 @@ def main():
     flops_dense = dense_flops(wl.batch, wl.n_heads, wl.seqlen, wl.head_dim)
     density = flops_sparse / flops_dense
 
-    clocks = ClockSampler(local, os.path.join(ROOT, "gpurun_out" if os.path.isdir(os.path.join(ROOT, "gpurun_out"))
-                                              else ".", f".clocks_rank{rank}.csv"))
+    clocks = ClockSampler(local, os.path.join(args.clocks_dir or tempfile.gettempdir(), f"wise_clocks_rank{rank}.csv"))
     time.sleep(0.3)
 
     # ---- timed: K trajectories
