@@ -272,6 +272,17 @@ int wise_support_overlap(const wise_shape_t* shape, const int32_t* idx_a, const 
  * when both were recorded), or WISE_ERR_CUDA if the synchronization failed. */
 int wise_get_status(cudaStream_t stream);
 
+/* Sets the time limit of each internal wait of the attention kernels
+ * (wise_full_attn_accumulate, its _noalloc variant, wise_sparse_attn and
+ * wise_freeze_a_attn) for every later launch in this process; ns == 0
+ * restores the default of 2 s.  A wait that runs out makes the kernel stop
+ * issuing work, let the work already in flight finish, and record
+ * WISE_ERR_TIMEOUT for wise_get_status(); the outputs of that launch are then
+ * incomplete.  The waits of that unwinding keep the 2 s limit.  Process-wide
+ * (not per device or stream); always returns WISE_OK.  The paper has no
+ * counterpart: this is the failure-detection control of the kernels. */
+int wise_set_wait_limit_ns(unsigned long long ns);
+
 /* Static description of a status code. */
 const char* wise_status_string(int status);
 

@@ -76,16 +76,11 @@
 #include <limits.h>
 #include <stdint.h>
 
+#include "attn_common.cuh"
 #include "internal.cuh"
 #include "ptx.cuh"
 
 namespace wise {
-
-// Key tiles are 128 keys wide whatever the block size: a tcgen05 MMA issued by
-// one thread costs about the same issue time at N = 32, 64 or 128, so narrower
-// tiles only waste tensor throughput.  Blocks of 32 or 64 are sub-blocks of a
-// tile, selected per (query block, key block) by the tile's mask.
-constexpr int kTileN = 128;
 
 template <int D>
 struct AttnCfg {
@@ -127,200 +122,6 @@ struct AttnCfg {
   static_assert(256 * kRegsSoftmax + 128 * kRegsOther <= kThreads * 168, "register split");
 };
 
-// Tile schedule rings.  Entry = {key tile | mask << 16, unit, flags, tile
-// index within its unit} (for the end marker: {0, 0, kEntEnd, number of
-// tiles}).  With S = 128 / block query blocks per query tile and key blocks
-// per key tile, bit qi * S + ki of the mask says that query block qi of the
-// tile attends key block ki of the key tile.  Flag bits 8 and up hold the
-// index of the unit among this CTA's units with tiles.
-constexpr int kSchedSlots = 16;  // per ring
-constexpr int kEntFirst = 4;     // first tile of its unit
-constexpr int kEntLast = 8;      // last tile of its unit
-constexpr int kEntEmpty = 16;    // unit without tiles (its output rows are zero)
-constexpr int kEntEnd = 32;      // no more units for this CTA
-constexpr int kEntUnitShift = 8;
-constexpr int kMmaRing = 2;  // ring of the two MMA threads
-
-__device__ __forceinline__ float ex2_approx(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-
-__device__ __forceinline__ float lg2_approx(float x) {
-  float y;
-  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-
-__device__ __forceinline__ float fmax3(float a, float b, float c) {
-  float d;
-  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
-  return d;
-}
-
-// Maximum of n values with a tree of three-input max operations.
-template <int N>
-__device__ __forceinline__ float row_max(const float (&s)[N]) {
-  float m[8];
-#pragma unroll
-  for (int e = 0; e < 8; ++e) m[e] = s[e];
-#pragma unroll
-  for (int c = 8; c + 1 < N; c += 16) {
-#pragma unroll
-    for (int e = 0; e < 8; ++e) m[e] = fmax3(m[e], s[c + e], (c + 8 + e < N) ? s[c + 8 + e] : s[c + e]);
-  }
-  return fmaxf(fmax3(m[0], m[1], m[2]), fmax3(fmax3(m[3], m[4], m[5]), m[6], m[7]));
-}
-
-// p = 2^(s * scale - shift) in place, two elements per packed FMA; returns
-// the sum of p.
-template <int N>
-__device__ __forceinline__ float exp2_scaled(float (&s)[N], float scale, float shift) {
-  const float2 sc = make_float2(scale, scale), sh = make_float2(-shift, -shift);
-  float2 acc[4];
-#pragma unroll
-  for (int e = 0; e < 4; ++e) acc[e] = make_float2(0.0f, 0.0f);
-#pragma unroll
-  for (int c = 0; c < N; c += 2) {
-    const float2 x = __ffma2_rn(make_float2(s[c], s[c + 1]), sc, sh);
-    const float2 y = make_float2(ex2_approx(x.x), ex2_approx(x.y));
-    s[c] = y.x;
-    s[c + 1] = y.y;
-    acc[(c / 2) & 3] = __fadd2_rn(acc[(c / 2) & 3], y);
-  }
-  const float2 b = __fadd2_rn(__fadd2_rn(acc[0], acc[1]), __fadd2_rn(acc[2], acc[3]));
-  return b.x + b.y;
-}
-
-// exp2_scaled that also returns the sums of the S column groups of N / S
-// columns (the key sub-blocks of a tile), for the block masses; S = 2 or 4.
-template <int N, int S>
-__device__ __forceinline__ float exp2_scaled_groups(float (&s)[N], float scale, float shift, float (&g)[S]) {
-  static_assert(S == 2 || S == 4, "groups");
-  constexpr int kChains = 4 / S;  // independent accumulation chains per group
-  constexpr int kCols = N / S;
-  const float2 sc = make_float2(scale, scale), sh = make_float2(-shift, -shift);
-  float2 acc[4];
-#pragma unroll
-  for (int e = 0; e < 4; ++e) acc[e] = make_float2(0.0f, 0.0f);
-#pragma unroll
-  for (int c = 0; c < N; c += 2) {
-    const float2 x = __ffma2_rn(make_float2(s[c], s[c + 1]), sc, sh);
-    const float2 y = make_float2(ex2_approx(x.x), ex2_approx(x.y));
-    s[c] = y.x;
-    s[c + 1] = y.y;
-    const int a = (c / kCols) * kChains + (c / 2) % kChains;
-    acc[a] = __fadd2_rn(acc[a], y);
-  }
-  float total = 0.0f;
-#pragma unroll
-  for (int k = 0; k < S; ++k) {
-    float2 t = acc[k * kChains];
-#pragma unroll
-    for (int ch = 1; ch < kChains; ++ch) t = __fadd2_rn(t, acc[k * kChains + ch]);
-    g[k] = t.x + t.y;
-    total += g[k];
-  }
-  return total;
-}
-
-// Key tiles of one unit in ascending order, with their sub-block masks
-// (S = 128 / BLK).  Dense: tiles 0..last, every sub-block (the causal limit is
-// applied per row).  Sparse: the merge of the support lists of the unit's S
-// query blocks; key block kb lies in key tile kb / S.  Entries that are
-// negative, beyond their query block, or not strictly ascending are skipped
-// and flagged in `bad`.  Fields a variant does not use are never touched, so
-// they cost no registers.
-template <int BLK, int MODE>
-struct TileIter {
-  static constexpr int S = kTileN / BLK;
-  int cur, last;             // dense
-  const int32_t* l0;         // sparse: list of query block q0; list q at l0 + q * cap
-  int cap, q0;
-  int pos[S];                // list q: entries read (low 16 bits) and count (high 16 bits); cap < 2^16
-  int pend[S];               // next entry of list q (the last one accepted), INT_MAX when done
-  int bad;
-
-  // Next valid entry of list q after pend[q]: in [0, q0 + q] and above it.
-  __device__ __forceinline__ int pull(int q) {
-    const int prev = pend[q];
-    while ((pos[q] & 0xFFFF) < (pos[q] >> 16)) {
-      const int v = __ldg(l0 + (size_t)q * cap + (pos[q] & 0xFFFF));
-      ++pos[q];
-      if (v >= 0 && v <= q0 + q && v > prev) return v;
-      bad = 1;
-    }
-    return INT_MAX;
-  }
-
-  __device__ __forceinline__ bool next(int& kt, uint32_t& mask) {
-    if constexpr (MODE != kSparse) {
-      if (cur > last) return false;
-      kt = cur++;
-      mask = S == 1 ? 1u : S == 2 ? 0xFu : 0xFFFFu;
-      return true;
-    } else {
-      int lo = pend[0];
-#pragma unroll
-      for (int q = 1; q < S; ++q) lo = min(lo, pend[q]);
-      if (lo == INT_MAX) return false;
-      kt = lo / S;
-      mask = 0;
-#pragma unroll
-      for (int q = 0; q < S; ++q) {
-        while (pend[q] != INT_MAX && pend[q] / S == kt) {
-          mask |= 1u << (q * S + pend[q] % S);
-          pend[q] = pull(q);
-        }
-      }
-      return true;
-    }
-  }
-};
-
-__device__ __forceinline__ int clamp_count(int n, int cap, int& bad) {
-  if (n < 0 || n > cap) {
-    bad = 1;
-    return n < 0 ? 0 : cap;
-  }
-  return n;
-}
-
-template <int BLK, int MODE>
-__device__ __forceinline__ TileIter<BLK, MODE> make_iter(const AttnParams& p, int b, int kvh, int qt) {
-  TileIter<BLK, MODE> it;
-  it.bad = 0;
-  if constexpr (MODE != kSparse) {
-    it.cur = 0;
-    const int last_row = min(qt * 128 + 127, p.seqlen - 1);
-    it.last = last_row / kTileN;
-  } else {
-    constexpr int S = TileIter<BLK, MODE>::S;
-    const int q0 = qt * S;
-    const size_t row0 = ((size_t)b * p.n_kv_heads + kvh) * p.n_blocks + q0;
-    it.l0 = p.idx + row0 * p.cap;
-    it.cap = p.cap;
-    it.q0 = q0;
-#pragma unroll
-    for (int q = 0; q < S; ++q) {
-      it.pos[q] = ((q0 + q < p.n_blocks) ? clamp_count(__ldg(p.counts + row0 + q), p.cap, it.bad) : 0) << 16;
-      it.pend[q] = -1;
-    }
-#pragma unroll
-    for (int q = 0; q < S; ++q) it.pend[q] = it.pull(q);
-  }
-  return it;
-}
-
-__device__ __forceinline__ void decode_unit(const AttnParams& p, int u, int& b, int& h, int& qt) {
-  const int bh_count = p.batch * p.n_heads;
-  qt = p.n_qtiles - 1 - u / bh_count;  // longest causal prefix first
-  const int bh = u % bh_count;
-  b = bh / p.n_heads;
-  h = bh % p.n_heads;
-}
-
 template <int RK, int RV>
 struct SharedState {
   uint64_t k_full[RK], k_empty[RK], v_full[RV], v_empty[RV];
@@ -352,17 +153,6 @@ struct SharedState {
   int abort;
 };
 
-// mbar_wait whose outcome is the same for every lane of the warp (all lanes
-// must call it together): a lane that gave up makes the whole warp give up.
-__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
-  return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort));
-}
-
-__device__ __forceinline__ void raise_status(const AttnParams& p, int* abort, int bits) {
-  *reinterpret_cast<volatile int*>(abort) = 1;
-  atomicOr(p.status, bits);
-}
-
 // ------------------------------------------------------------------ producer
 template <int D, int BLK, int MODE>
 __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, const CUtensorMap* mapV,
@@ -383,7 +173,7 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
     const int e = ring_w == kMmaRing ? jt : ring_w == 1 ? (jt >> 1) : ((jt + 1) >> 1) + n_empty;
     const int slot = e % kSchedSlots;
     if (e >= kSchedSlots &&
-        !mbar_wait(&sb.sched_empty[ring_w][slot], ((e / kSchedSlots) - 1) & 1, abort))
+        !mbar_wait(&sb.sched_empty[ring_w][slot], ((e / kSchedSlots) - 1) & 1, abort, p.wait_ns))
       return false;
     sb.sched[ring_w][slot] = make_int4(kb, u, flags, t);
     mbar_arrive(&sb.sched_full[ring_w][slot]);  // release: the entry is visible to whoever acquires the phase
@@ -392,7 +182,7 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
   auto load = [&](const CUtensorMap* map, uint8_t* base, uint64_t* full, uint64_t* empty, int R, int& j, int kb,
                   int z) -> bool {
     const int slot = j % R;
-    if (j >= R && !mbar_wait(&empty[slot], ((j / R) - 1) & 1, abort)) return false;
+    if (j >= R && !mbar_wait(&empty[slot], ((j / R) - 1) & 1, abort, p.wait_ns)) return false;
     mbar_arrive_expect_tx(&full[slot], C::kKVBytes);
     for (int i = 0; i < C::kBoxes; ++i)
       tma_load_3d(base + slot * C::kKVBytes + i * kTileN * 128, map, &full[slot], 64 * i, kb * kTileN, z);
@@ -432,7 +222,7 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
       ++jt;
       if (first) {
         // The staging buffer is free once the previous unit's Q is in TMEM.
-        if (nq >= 1 && !mbar_wait(&sb.q_stage_free, (nq - 1) & 1, abort)) {
+        if (nq >= 1 && !mbar_wait(&sb.q_stage_free, (nq - 1) & 1, abort, p.wait_ns)) {
           ok = false;
           break;
         }
@@ -476,9 +266,9 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
 
 // Single thread: reads entry e of the MMA ring (tile e, or the end marker).
 template <class SS>
-__device__ __forceinline__ bool sched_read_mma(SS& sb, int e, int4& ent, volatile int* abort) {
+__device__ __forceinline__ bool sched_read_mma(SS& sb, int e, int4& ent, volatile int* abort, uint64_t limit_ns) {
   const int slot = e % kSchedSlots;
-  if (!mbar_wait(&sb.sched_full[kMmaRing][slot], (e / kSchedSlots) & 1, abort)) return false;
+  if (!mbar_wait(&sb.sched_full[kMmaRing][slot], (e / kSchedSlots) & 1, abort, limit_ns)) return false;
   ent = sb.sched[kMmaRing][slot];
   mbar_arrive(&sb.sched_empty[kMmaRing][slot]);
   return true;
@@ -496,18 +286,18 @@ __device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* q_stage,
   bool ok = true;
   for (;;) {
     int4 ent;
-    if (!sched_read_mma(sb, j, ent, abort)) {
+    if (!sched_read_mma(sb, j, ent, abort, p.wait_ns)) {
       ok = false;
       break;
     }
     if (ent.z & kEntEnd) break;
     if (ent.z & kEntFirst) {
       // Q in TMEM was last read by the S products of unit nq - 1.
-      if (nq >= 1 && !mbar_wait(&sb.q_free, (nq - 1) & 1, abort)) {
+      if (nq >= 1 && !mbar_wait(&sb.q_free, (nq - 1) & 1, abort, p.wait_ns)) {
         ok = false;
         break;
       }
-      if (!mbar_wait(&sb.q_full, nq & 1, abort)) {
+      if (!mbar_wait(&sb.q_full, nq & 1, abort, p.wait_ns)) {
         ok = false;
         break;
       }
@@ -521,12 +311,12 @@ __device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* q_stage,
       ++nq;
     }
     const int slot = j % RK;
-    if (!mbar_wait(&sb.k_full[slot], (j / RK) & 1, abort)) {
+    if (!mbar_wait(&sb.k_full[slot], (j / RK) & 1, abort, p.wait_ns)) {
       ok = false;
       break;
     }
     // S(j) overwrites S(j-1): its softmax warpgroup must have read it.
-    if (j >= 1 && !mbar_wait(&sb.s_free[(j - 1) & 1], ((j - 1) >> 1) & 1, abort)) {
+    if (j >= 1 && !mbar_wait(&sb.s_free[(j - 1) & 1], ((j - 1) >> 1) & 1, abort, p.wait_ns)) {
       ok = false;
       break;
     }
@@ -564,7 +354,7 @@ __device__ void attn_mma_pv(const AttnParams& p, uint32_t tmem, uint8_t* ring,
   bool ok = true;
   for (;;) {
     int4 ent;
-    if (!sched_read_mma(sb, j, ent, abort)) {
+    if (!sched_read_mma(sb, j, ent, abort, p.wait_ns)) {
       ok = false;
       break;
     }
@@ -573,18 +363,18 @@ __device__ void attn_mma_pv(const AttnParams& p, uint32_t tmem, uint8_t* ring,
     if (first) {
       // The first P V of a unit overwrites O: both epilogue halves of the
       // previous unit must have read it.
-      if (nu >= 1 && !mbar_wait(&sb.o_free, (nu - 1) & 1, abort)) {
+      if (nu >= 1 && !mbar_wait(&sb.o_free, (nu - 1) & 1, abort, p.wait_ns)) {
         ok = false;
         break;
       }
       ++nu;
     }
     const int slot = j % RV;
-    if (!mbar_wait(&sb.p_full[j & 1], (j >> 1) & 1, abort)) {
+    if (!mbar_wait(&sb.p_full[j & 1], (j >> 1) & 1, abort, p.wait_ns)) {
       ok = false;
       break;
     }
-    if (!mbar_wait(&sb.v_full[slot], (j / RV) & 1, abort)) {
+    if (!mbar_wait(&sb.v_full[slot], (j / RV) & 1, abort, p.wait_ns)) {
       ok = false;
       break;
     }
@@ -603,47 +393,6 @@ __device__ void attn_mma_pv(const AttnParams& p, uint32_t tmem, uint8_t* ring,
   umma_commit(&sb.pv_done);
   int never = 0;
   mbar_wait(&sb.pv_done, 0, &never);
-}
-
-// Loads N consecutive 32-bit TMEM columns of this thread's lane (N = 64, 96
-// or 128: 32-column loads issued together, one wait).
-template <int N>
-__device__ __forceinline__ void tmem_load_row(uint32_t addr, float (&x)[N]) {
-  static_assert(N == 64 || N == 96 || N == 128, "row width");
-  uint32_t va[32], vb[32], vc[32], vd[32];
-  tmem_ld_32x32b_x32(addr, va);
-  tmem_ld_32x32b_x32(addr + 32, vb);
-  if constexpr (N >= 96) tmem_ld_32x32b_x32(addr + 64, vc);
-  if constexpr (N == 128) tmem_ld_32x32b_x32(addr + 96, vd);
-  tmem_ld_wait(va, vb);  // completes every load issued above
-  if constexpr (N >= 96) reg_tie(vc);
-  if constexpr (N == 128) reg_tie(vd);
-#pragma unroll
-  for (int e = 0; e < 32; ++e) {
-    x[e] = __uint_as_float(va[e]);
-    x[32 + e] = __uint_as_float(vb[e]);
-    if constexpr (N >= 96) x[64 + e] = __uint_as_float(vc[e]);
-    if constexpr (N == 128) x[96 + e] = __uint_as_float(vd[e]);
-  }
-}
-
-// Loads this thread's row of an S tile (kTileN columns) and applies the
-// causal / support masks: column c of key sub-block k = c / BLK is kept if
-// bit k of `sub` is set and c <= lim (keys with c > lim are in the future of
-// this row).
-template <int BLK>
-__device__ __forceinline__ void load_s_row(uint32_t addr, float (&s)[kTileN], uint32_t sub, int lim) {
-  constexpr int S = kTileN / BLK;
-  tmem_load_row<kTileN>(addr, s);
-  if (sub != (1u << S) - 1u || lim < kTileN - 1) {
-    // Per sub-block limit: lim where the row attends the sub-block, else the
-    // column before it, so that a single compare masks the column.
-    int lim_k[S];
-#pragma unroll
-    for (int k = 0; k < S; ++k) lim_k[k] = ((sub >> k) & 1u) ? lim : k * BLK - 1;
-#pragma unroll
-    for (int c = 0; c < kTileN; ++c) s[c] = (c > lim_k[c / BLK]) ? -INFINITY : s[c];
-  }
 }
 
 // What the epilogue needs about its unit.
@@ -693,7 +442,7 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
   // ---- one tile (j & 1 == w): key tile and mask in `key`, tile t of the
   // unit with index unit_ix
   auto tile = [&](int key, bool first, int t, int unit_ix) -> bool {
-    if (!warp_wait(&sb.s_full[w], (j >> 1) & 1, abort)) return false;
+    if (!warp_wait(&sb.s_full[w], (j >> 1) & 1, abort, p.wait_ns)) return false;
     tc_fence_after_sync();
     const int kb = key & 0xFFFF;
     const uint32_t sub = ((uint32_t)key >> (16 + qsub * S)) & ((1u << S) - 1u);
@@ -709,7 +458,7 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     float m_prev = -INFINITY;
     if (!first) {
       const int jp = j - 1;
-      if (!warp_wait(&sb.m_pub[w ^ 1][(jp >> 1) & 1], (jp >> 2) & 1, abort)) return false;
+      if (!warp_wait(&sb.m_pub[w ^ 1][(jp >> 1) & 1], (jp >> 2) & 1, abort, p.wait_ns)) return false;
       m_prev = sb.mx[w ^ 1][(jp >> 1) & 1][r];
     }
     const float m_new = (m_tile > m_prev + kRescaleThreshold) ? m_tile : m_prev;
@@ -730,7 +479,7 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     for (int e = 0; e < kTileN / 2; ++e) pw[e] = pack_bf16x2(s[2 * e], s[2 * e + 1]);
     // P buffer w was last read by P V(j-2); this warpgroup waited for P V(j-4)
     // at its previous tile, so o_full[w] is at most one phase short.
-    if (j >= 2 && !warp_wait(&sb.o_full[w], ((j >> 1) - 1) & 1, abort)) return false;
+    if (j >= 2 && !warp_wait(&sb.o_full[w], ((j >> 1) - 1) & 1, abort, p.wait_ns)) return false;
     tc_fence_after_sync();
     // The stores complete while the bookkeeping below runs.
 #pragma unroll
@@ -760,7 +509,7 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     const bool rescale = !first && m_new != m_prev && m_prev != -INFINITY;
     if (__any_sync(0xffffffffu, rescale)) {
       // O must have received P V(j-1); P V(j-3) completed (the wait above).
-      if (!warp_wait(&sb.o_full[(j - 1) & 1], ((j - 1) >> 1) & 1, abort)) return false;
+      if (!warp_wait(&sb.o_full[(j - 1) & 1], ((j - 1) >> 1) & 1, abort, p.wait_ns)) return false;
       tc_fence_after_sync();
       const float f = rescale ? ex2_approx(m_prev - m_new) : 1.0f;
 #pragma unroll
@@ -783,7 +532,7 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
   // ---- the epilogue, run by L (this warpgroup handled the unit's last tile)
   auto epilogue = [&](const EpiInfo& ei) -> bool {
     const int x = w ^ 1;  // E
-    if (!warp_wait(&sb.l_pub[x], n_epi & 1, abort)) return false;
+    if (!warp_wait(&sb.l_pub[x], n_epi & 1, abort, p.wait_ns)) return false;
     const float lE = sb.lx[x][r], mE = sb.lm[x][r];
     __syncwarp();
     if (lane == 0) mbar_arrive(&sb.l_ack[x]);
@@ -792,7 +541,7 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     const float l_row = (mE == -INFINITY) ? ei.l : ei.l + lE * ex2_approx(mE - ei.m);
     // P V(j1-2) completed before P(j1) was written, so o_full[j1 & 1] is at
     // most one phase short of P V(j1).
-    if (!warp_wait(&sb.o_full[ei.j1 & 1], (ei.j1 >> 1) & 1, abort)) return false;
+    if (!warp_wait(&sb.o_full[ei.j1 & 1], (ei.j1 >> 1) & 1, abort, p.wait_ns)) return false;
     tc_fence_after_sync();
     float o[D];
     tmem_load_row<D>(lane_tmem + C::kTmemO, o);
@@ -849,7 +598,7 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
       // acquire at CTA scope).
       __syncwarp();
       if (lane == 0) mbar_arrive(&sb.epi[w]);
-      if (!warp_wait(&sb.epi[w], n_epi & 1, abort)) return false;
+      if (!warp_wait(&sb.epi[w], n_epi & 1, abort, p.wait_ns)) return false;
       constexpr int kWarpsPerBlock = BLK / 32;  // warps holding one query block's rows
       const float inv_b = 1.0f / (float)BLK;
       for (int e = r; e < S * p.n_blocks; e += 128) {
@@ -876,7 +625,7 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
   // ended (zero if this warpgroup handled none of its tiles), once L has read
   // the previous one.
   auto publish = [&]() -> bool {
-    if (n_pub >= 1 && !warp_wait(&sb.l_ack[w], (n_pub - 1) & 1, abort)) return false;
+    if (n_pub >= 1 && !warp_wait(&sb.l_ack[w], (n_pub - 1) & 1, abort, p.wait_ns)) return false;
     sb.lx[w][r] = fresh ? 0.0f : l_w;
     sb.lm[w][r] = fresh ? -INFINITY : m_w;
     // The staging boxes are shared by the two warpgroups and a bulk-group
@@ -893,7 +642,7 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
 
   for (;;) {
     const int slot = pos % kSchedSlots;
-    if (!warp_wait(&sb.sched_full[w][slot], (pos / kSchedSlots) & 1, abort)) {
+    if (!warp_wait(&sb.sched_full[w][slot], (pos / kSchedSlots) & 1, abort, p.wait_ns)) {
       ok = false;
       break;
     }

@@ -40,6 +40,7 @@ struct AttnParams {
   int cap;                // kSparse
   float* scratch;         // kDenseMass: scratch_floats_per_cta(n_blocks) floats per CTA
   int* status;
+  unsigned long long wait_ns;  // limit of each bounded wait on the main path (kWaitLimitNs by default)
 };
 
 struct AttnLaunch {

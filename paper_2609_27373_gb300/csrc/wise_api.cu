@@ -4,11 +4,13 @@
 #include <string.h>
 
 #include <algorithm>
+#include <atomic>
 #include <math.h>
 #include <mutex>
 
 #include "wise.h"
 #include "internal.cuh"
+#include "ptx.cuh"
 
 namespace wise {
 namespace {
@@ -29,6 +31,10 @@ struct DeviceState {
 
 std::mutex g_mutex;
 DeviceState g_dev[kMaxDevices];
+
+// Limit of each bounded wait inside the attention kernels, taken by every
+// later launch (wise_set_wait_limit_ns).
+std::atomic<unsigned long long> g_wait_ns{kWaitLimitNs};
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
@@ -179,6 +185,7 @@ int launch_attention(const wise_shape_t* sh, const void* Q, const void* K, const
   p.counts = counts;
   p.cap = cap;
   p.status = ds->status;
+  p.wait_ns = g_wait_ns.load(std::memory_order_relaxed);
   L.grid = (int)(units < ds->sm_count ? units : ds->sm_count);
   L.stream = stream;
   p.scratch = nullptr;
@@ -469,6 +476,11 @@ extern "C" const char* wise_status_string(int status) {
     case WISE_ERR_BAD_SUPPORT: return "support list entries out of range, unordered or over cap";
     default: return "unknown status";
   }
+}
+
+extern "C" int wise_set_wait_limit_ns(unsigned long long ns) {
+  g_wait_ns.store(ns == 0 ? kWaitLimitNs : ns, std::memory_order_relaxed);
+  return WISE_OK;
 }
 
 extern "C" int wise_version(void) { return 100; }

@@ -29,7 +29,8 @@ WISE_SEL_COVERAGE = 1
 EXPORTS = ("wise_full_attn_accumulate", "wise_full_attn_accumulate_noalloc", "wise_select_support",
            "wise_sparse_attn", "wise_freeze_a_attn", "wise_freeze_a_probs", "wise_frozen_pv", "wise_support_mass",
            "wise_support_overlap",
-           "wise_select_working_set", "wise_get_status", "wise_status_string", "wise_version")
+           "wise_select_working_set", "wise_get_status", "wise_set_wait_limit_ns", "wise_status_string",
+           "wise_version")
 NOALLOC_SCRATCH_BYTES = 8 << 20
 
 
@@ -113,6 +114,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.wise_select_working_set.argtypes = [ctypes.POINTER(wise_shape_t), I, ctypes.c_float, I, I, P, I, P, P,
                                                 I, P, P, I, P]
         lib.wise_get_status.argtypes = [P]
+        lib.wise_set_wait_limit_ns.argtypes = [ctypes.c_ulonglong]
         lib.wise_status_string.argtypes = [ctypes.c_int]
         lib.wise_status_string.restype = ctypes.c_char_p
         lib.wise_version.restype = ctypes.c_int
@@ -361,6 +363,15 @@ def wise_select_working_set(shape: Shape, mode: int, step_masses, idx, counts, e
 def wise_get_status(stream=None) -> int:
     """Synchronizes the stream and returns (and clears) the device status word."""
     return int(load().wise_get_status(_stream(stream)))
+
+
+def wise_set_wait_limit_ns(ns: int) -> None:
+    """Limit of each internal wait of the attention kernels for later launches (0 = the 2 s default)."""
+    if ns < 0:
+        raise ValueError("ns must be >= 0")
+    rc = load().wise_set_wait_limit_ns(int(ns))
+    if rc != WISE_OK:
+        raise WiseError(rc, "wise_set_wait_limit_ns")
 
 
 def wise_version() -> int:
