@@ -130,11 +130,14 @@ int wise_full_attn_accumulate(const wise_shape_t* shape, const void* Q, const vo
  * bytes of scratch (nT/2 rounded down); larger problems return
  * WISE_ERR_UNSUPPORTED and launch nothing.  On a 152-SM GB300 with at least
  * 152 query tiles that is nT <= 49 with block 128 (seqlen <= 6272).
- * The first call on each device looks up the array's device address (with
- * that device current) and caches it; make that first call before any CUDA
- * stream capture.  All calls on a device share the one array: calls whose
- * kernels can run at the same time on that device (unordered streams) race
- * on it and corrupt each other's block mass. */
+ * The first call on each device that passes the argument checks looks up
+ * the array's device address (with that device current) and caches it; make
+ * that first call before any CUDA stream capture.  The cached address is not
+ * refreshed: calls must not span a cudaDeviceReset of the device.  All calls
+ * on a device share the one array: calls whose kernels can run at the same
+ * time on that device (unordered streams) race on it and corrupt each other's
+ * block mass.  Argument checks and error codes are those of
+ * wise_full_attn_accumulate (blockmass == NULL is WISE_ERR_INVALID_ARG). */
 int wise_full_attn_accumulate_noalloc(const wise_shape_t* shape, const void* Q, const void* K, const void* V,
                                       void* O, float* blockmass, int step, cudaStream_t stream);
 

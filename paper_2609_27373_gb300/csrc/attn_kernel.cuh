@@ -700,7 +700,10 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     }
     j += 2;
   }
-  // Output stores issued by this warp must complete before the CTA exits.
+  // A warp that gave up inside a tile may still have TMEM stores in flight:
+  // they complete before TMEM is released.  Output stores issued by this
+  // warp complete before the CTA exits.
+  tmem_st_wait();
   if (lane == 0) tma_store_wait_all();
   if (!ok) raise_status(p, &sb.abort, kStatusTimeout);
 }

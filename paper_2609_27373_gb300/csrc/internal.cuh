@@ -67,12 +67,18 @@ struct SelectParams {
 
 // Argument checks, tensor maps and launch of the attention kernels (defined
 // in wise_api.cu).  For kDenseMass the per-CTA scratch comes from the
-// library's lazily allocated per-device buffer, unless caller_scratch is
-// given: then that device buffer of caller_scratch_bytes is used and a
-// problem needing more returns WISE_ERR_UNSUPPORTED.
+// library's lazily allocated per-device buffer, unless fixed_scratch is set:
+// then it is the fixed array of noalloc.cu (its address resolved by
+// noalloc_scratch_address once the arguments and the device have been
+// checked), and a problem needing more than WISE_NOALLOC_SCRATCH_BYTES
+// returns WISE_ERR_UNSUPPORTED.
 int launch_attention(const wise_shape_t* sh, const void* Q, const void* K, const void* V, void* O, int mode,
                      float* blockmass, int step, const int32_t* idx, const int32_t* counts, int cap,
-                     cudaStream_t stream, float* caller_scratch = nullptr, size_t caller_scratch_bytes = 0);
+                     cudaStream_t stream, bool fixed_scratch = false);
+
+// Device address of the fixed scratch array on the current device (looked up
+// once per device and cached; defined in noalloc.cu).
+int noalloc_scratch_address(float** out);
 
 // Defined in select.cu.
 cudaError_t launch_select(const SelectParams& p, cudaStream_t stream);

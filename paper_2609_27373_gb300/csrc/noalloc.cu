@@ -14,15 +14,17 @@
 static __device__ __align__(256) float wise_noalloc_scratch[WISE_NOALLOC_SCRATCH_BYTES / sizeof(float)];
 
 namespace wise {
-namespace {
 
+namespace {
 constexpr int kMaxDevices = 64;
 std::mutex g_noalloc_mutex;
 float* g_noalloc_scratch_ptr[kMaxDevices];
+}  // namespace
 
-// Device address of the scratch array on the current device.  In host code
-// the array's name only stands for the symbol; the address a kernel can use
-// is looked up once per device, with that device current, and cached.
+// In host code the array's name only stands for the symbol; the address a
+// kernel can use is looked up once per device, with that device current, and
+// cached.  The cache is not invalidated: calls must not span a
+// cudaDeviceReset of the device (which unloads the module holding the array).
 int noalloc_scratch_address(float** out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return WISE_ERR_CUDA;
@@ -36,17 +38,14 @@ int noalloc_scratch_address(float** out) {
   return WISE_OK;
 }
 
-}  // namespace
 }  // namespace wise
 
 extern "C" int wise_full_attn_accumulate_noalloc(const wise_shape_t* shape, const void* Q, const void* K,
                                                  const void* V, void* O, float* blockmass, int step,
                                                  cudaStream_t stream) {
-  if (!shape || !blockmass) return WISE_ERR_INVALID_ARG;
-  if (shape->batch == 0 || shape->seqlen == 0) return WISE_OK;
-  float* scratch = nullptr;
-  const int rc = wise::noalloc_scratch_address(&scratch);
-  if (rc != WISE_OK) return rc;
+  // The shape, pointers and device are checked exactly as for
+  // wise_full_attn_accumulate before the array's address is resolved.
+  if (!blockmass) return WISE_ERR_INVALID_ARG;
   return wise::launch_attention(shape, Q, K, V, O, wise::kDenseMass, blockmass, step, nullptr, nullptr, 0, stream,
-                                scratch, sizeof(wise_noalloc_scratch));
+                                /*fixed_scratch=*/true);
 }

@@ -138,7 +138,7 @@ bool make_map(CUtensorMap* map, const void* base, int head_dim, int seqlen, long
 
 int launch_attention(const wise_shape_t* sh, const void* Q, const void* K, const void* V, void* O, int mode,
                      float* blockmass, int step, const int32_t* idx, const int32_t* counts, int cap,
-                     cudaStream_t stream, float* caller_scratch, size_t caller_scratch_bytes) {
+                     cudaStream_t stream, bool fixed_scratch) {
   int rc = check_shape(sh, true);
   if (rc != WISE_OK) return rc;
   if (sh->batch == 0 || sh->seqlen == 0) return WISE_OK;
@@ -193,9 +193,10 @@ int launch_attention(const wise_shape_t* sh, const void* Q, const void* K, const
     // Per CTA: log2 partial masses per key sub-block and per-warp sums.
     const size_t need =
         (size_t)L.grid * scratch_floats_per_cta(p.n_qtiles, 128 / sh->block, n_blocks) * sizeof(float);
-    if (caller_scratch) {
-      if (need > caller_scratch_bytes) return WISE_ERR_UNSUPPORTED;
-      p.scratch = caller_scratch;
+    if (fixed_scratch) {
+      if (need > WISE_NOALLOC_SCRATCH_BYTES) return WISE_ERR_UNSUPPORTED;
+      const int rs = noalloc_scratch_address(&p.scratch);
+      if (rs != WISE_OK) return rs;
     } else {
       p.scratch = scratch_at_least(ds, need);
       if (!p.scratch) return WISE_ERR_CUDA;

@@ -71,6 +71,26 @@ def test_empty_problems_are_a_no_op():
         assert lib.wise_sparse_attn(ctypes.byref(sh), NULL, NULL, NULL, NULL, NULL, 4, NULL, NULL) == 0
 
 
+@pytest.mark.parametrize("kw,code", [
+    (dict(block=16), wise.WISE_ERR_UNSUPPORTED),
+    (dict(head_dim=80), wise.WISE_ERR_UNSUPPORTED),
+    (dict(seqlen=200), wise.WISE_ERR_SHAPE),
+    (dict(batch=0, block=16), wise.WISE_ERR_UNSUPPORTED),   # empty, but still an invalid shape
+    (dict(seqlen=0, head_dim=80), wise.WISE_ERR_UNSUPPORTED),
+    (dict(batch=0), wise.WISE_OK),                           # empty and valid: a no-op
+])
+def test_noalloc_entry_point_checks_like_the_allocating_one(kw, code):
+    # The same checks, in the same order, as wise_full_attn_accumulate with a
+    # block-mass buffer (all of them run before any device is touched).
+    lib = wise.load()
+    sh = _shape(**kw)
+    mass = ctypes.c_void_p(0x1000)
+    assert lib.wise_full_attn_accumulate(ctypes.byref(sh), NULL, NULL, NULL, NULL, mass, 0, NULL) == code
+    assert lib.wise_full_attn_accumulate_noalloc(ctypes.byref(sh), NULL, NULL, NULL, NULL, mass, 0, NULL) == code
+    assert lib.wise_full_attn_accumulate_noalloc(ctypes.byref(sh), NULL, NULL, NULL, NULL, NULL, 0, NULL) == \
+        wise.WISE_ERR_INVALID_ARG
+
+
 def test_misaligned_pointer_is_rejected():
     lib = wise.load()
     sh = _shape()

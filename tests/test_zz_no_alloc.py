@@ -11,6 +11,11 @@ step that overwrites the mass and a second that accumulates), and refuse a
 problem whose scratch would not fit.  This file is collected last so that a
 run stopping at its first failure has already run every other test.
 """
+import os
+import subprocess
+import sys
+import textwrap
+
 import numpy as np
 import pytest
 import torch
@@ -55,3 +60,44 @@ def test_noalloc_rejects_a_problem_beyond_its_scratch():
         wise.wise_full_attn_accumulate_noalloc(shape, Q, K, K, O, mass, 0)
     assert e.value.code == wise.WISE_ERR_UNSUPPORTED
     assert wise.wise_get_status() == wise.WISE_OK
+
+
+_FRESH_PROCESS = textwrap.dedent("""
+    import sys, torch
+    sys.path.insert(0, sys.argv[1])
+    from paper_2609_27373_gb300 import synth, wise
+    wise.load()
+    B, H, L, D, blk = 1, 8, 2048, 128, 128
+    shape = wise.Shape(B, L, H, H, D, blk)
+    nb = shape.n_blocks
+    to = lambda x: torch.from_numpy(x.view("int16")).view(torch.bfloat16).cuda()
+    Q, K, V = (to(x) for x in synth.random_qkv(B, H, H, L, D, seed=3))
+    O = torch.empty_like(Q)
+    mass = torch.zeros((B, H, nb, nb), dtype=torch.float32, device="cuda")
+    torch.cuda.synchronize()
+    # Plain dense attention (no scratch) loads the library's module first.
+    wise.wise_full_attn_accumulate(shape, Q, K, V, O)
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    for step in range(3):
+        wise.wise_full_attn_accumulate_noalloc(shape, Q, K, V, O, mass, step)
+    torch.cuda.synchronize()
+    free1 = torch.cuda.mem_get_info()[0]
+    print(free0, free1, wise.wise_get_status())
+""")
+
+
+def test_noalloc_allocates_nothing_in_a_fresh_process():
+    # A fresh process whose first block-mass calls are the no-allocation
+    # ones: free device memory must not change across them.  (The allocating
+    # entry point would take its scratch, several MiB, with cudaMalloc on its
+    # first call; modules are loaded eagerly so that loading a kernel is not
+    # mistaken for an allocation.)
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = dict(os.environ, CUDA_MODULE_LOADING="EAGER")
+    r = subprocess.run([sys.executable, "-c", _FRESH_PROCESS, root], capture_output=True, text=True, env=env,
+                       timeout=600)
+    assert r.returncode == 0, r.stderr[-2000:]
+    free0, free1, status = (int(x) for x in r.stdout.split()[-3:])
+    assert status == wise.WISE_OK
+    assert free1 == free0, f"device memory changed by {free0 - free1} bytes across the no-allocation calls"
