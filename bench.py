@@ -225,14 +225,15 @@ def run_reference(args):
 
 # --------------------------------------------------------------------------- GPU arm
 
-def run_profile_sequence():
+def run_profile_sequence(name=WORKLOAD):
     """Fixed launch sequence for profilers: n_discovery dense+mass launches,
-    one selection, two sparse launches, one plain dense launch, one Freeze-A
-    store and two stored-Freeze-A P V launches of the 4K workload (about 1 GB
-    on the device)."""
+    one selection, two sparse launches and one plain dense launch of a
+    workload, then (4K workload only) one Freeze-A store and two
+    stored-Freeze-A P V launches (about 1 GB on the device at 4K, under 1.5 GB
+    for the other workloads)."""
     import torch
     from paper_2609_27373_gb300 import synth, wise
-    wl = synth.WORKLOADS[WORKLOAD]
+    wl = synth.WORKLOADS[name]
     shape, sel = wise.shape_of(wl), wise.select_of(wl)
     layer = wise.WiseAttention(shape, sel, wl.n_discovery)
     traj = synth.Trajectory(wl)
@@ -242,6 +243,11 @@ def run_profile_sequence():
         layer.step(t, Q, K, V, O)
     wise.wise_sparse_attn(shape, Q, K, V, layer.idx, layer.counts, O)
     wise.wise_full_attn_accumulate(shape, Q, K, V, O)
+    if name != WORKLOAD:
+        status = wise.wise_get_status()
+        if status != wise.WISE_OK:
+            raise RuntimeError(wise.status_string(status))
+        return 0
     # Freeze-A with the distribution stored once, then two late-step P V launches
     n_units = wl.batch * wl.n_heads * (wl.seqlen // 128)
     P = torch.empty((n_units, wise.freeze_tile_cap(shape, wl.cap), 128, 128), dtype=torch.bfloat16, device="cuda")
@@ -267,13 +273,15 @@ def main():
     ap.add_argument("--profile", action="store_true",
                     help="no timing: the 4K discovery steps, one selection, then 2 late sparse and 1 dense launches "
                          "(a small, fixed launch sequence for ncu captures)")
+    ap.add_argument("--profile-workload", default=WORKLOAD,
+                    help="workload of --profile (4k, 4k_b32, 4k_b4_d96, 16k, 32k_gqa, tiny)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("at least 3 warm-up steps")
     if args.impl == "reference":
         return run_reference(args)
     if args.profile:
-        return run_profile_sequence()
+        return run_profile_sequence(args.profile_workload)
 
     import torch
     import torch.distributed as dist

@@ -206,10 +206,25 @@ __device__ __forceinline__ TileIter<BLK, MODE> make_iter(const AttnParams& p, in
   return it;
 }
 
+// Unit u -> (batch, head, query tile).  Units are numbered by decreasing
+// causal length (the grid deals them out in a snake order that evens out the
+// per-CTA sums).  With group_heads > 0 the (batch, head) pairs are taken in
+// groups of group_heads consecutive ones (whole kv-head groups), all units of
+// a group before the next, so that the K and V of a group stay in L2 while
+// all its query tiles read them.
 __device__ __forceinline__ void decode_unit(const AttnParams& p, int u, int& b, int& h, int& qt) {
   const int bh_count = p.batch * p.n_heads;
-  qt = p.n_qtiles - 1 - u / bh_count;  // longest causal prefix first
-  const int bh = u % bh_count;
+  int bh;
+  if (p.group_heads > 0) {
+    const int per_group = p.group_heads * p.n_qtiles;
+    const int g = u / per_group, v = u - g * per_group;
+    const int gh = min(p.group_heads, bh_count - g * p.group_heads);  // the last group may be smaller
+    qt = p.n_qtiles - 1 - v / gh;
+    bh = g * p.group_heads + v % gh;
+  } else {
+    qt = p.n_qtiles - 1 - u / bh_count;
+    bh = u % bh_count;
+  }
   b = bh / p.n_heads;
   h = bh % p.n_heads;
 }

@@ -31,6 +31,7 @@ struct AttnParams {
   int n_qtiles;   // ceil(seqlen / 128): 128-row query tiles
   int n_blocks;   // nQB = nKB = seqlen / block
   int n_units;    // batch * n_heads * n_qtiles
+  int group_heads;  // unit order (decode_unit): 0 = by query tile over all heads, else heads in groups of this size
   float scale_log2;
   __nv_bfloat16* O;
   float* blockmass;       // kDenseMass

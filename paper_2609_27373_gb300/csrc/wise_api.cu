@@ -176,6 +176,21 @@ int launch_attention(const wise_shape_t* sh, const void* Q, const void* K, const
   const long long units = outer_q * p.n_qtiles;
   if (units > INT32_MAX) return WISE_ERR_UNSUPPORTED;
   p.n_units = (int)units;
+  // Unit order: when the K and V of all heads do not stay resident in L2
+  // (more than 64 MiB), heads are processed in equal groups of whole kv-head
+  // groups whose K and V take at most 48 MiB, so that each K/V tile is read
+  // from DRAM about once instead of once per wave of query tiles.
+  {
+    const double kv_bytes = (double)sh->seqlen * sh->head_dim * 2.0 * 2.0;  // K and V of one kv head
+    p.group_heads = 0;
+    if (kv_bytes * (double)outer_kv > 64.0 * (1 << 20)) {
+      long long g_kv = (long long)((48.0 * (1 << 20)) / kv_bytes);
+      if (g_kv < 1) g_kv = 1;
+      const long long n_groups = (outer_kv + g_kv - 1) / g_kv;
+      g_kv = (outer_kv + n_groups - 1) / n_groups;
+      p.group_heads = (int)(g_kv * p.group);
+    }
+  }
   const float scale = sh->scale > 0.0f ? sh->scale : 1.0f / sqrtf((float)sh->head_dim);
   p.scale_log2 = scale * 1.4426950408889634f;
   p.O = reinterpret_cast<__nv_bfloat16*>(O);
