@@ -252,6 +252,15 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
   if (ok && have_prev && !load(mapV, v_ring, sb.v_full, sb.v_empty, RV, jv, prev_kb, prev_z)) ok = false;
   for (int rw = 0; rw < 3 && ok; ++rw)
     if (!emit(rw, 0, 0, kEntEnd, jt)) ok = false;
+  // The MMA threads read tile j's entry of the MMA ring once K(j) (S thread)
+  // or V(j) (P V thread) has landed, the entry being written before either
+  // is loaded.  The end marker is announced the same way: the next K and V
+  // barriers complete without a copy, once their slots' last loads have been
+  // consumed.
+  if (ok && jk >= RK && !mbar_wait(&sb.k_empty[jk % RK], ((jk / RK) - 1) & 1, abort, p.wait_ns)) ok = false;
+  if (ok) mbar_arrive(&sb.k_full[jk % RK]);
+  if (ok && jv >= RV && !mbar_wait(&sb.v_empty[jv % RV], ((jv / RV) - 1) & 1, abort, p.wait_ns)) ok = false;
+  if (ok) mbar_arrive(&sb.v_full[jv % RV]);
   if (bad) atomicOr(p.status, kStatusBadSupport);
   if (!ok) {
     raise_status(p, &sb.abort, kStatusTimeout);
@@ -262,16 +271,6 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
     for (int t = max(0, jv - RV); t < jv; ++t) mbar_wait(&sb.v_full[t % RV], (t / RV) & 1, &never);
     if (nq > 0) mbar_wait(&sb.q_full, (nq - 1) & 1, &never);
   }
-}
-
-// Single thread: reads entry e of the MMA ring (tile e, or the end marker).
-template <class SS>
-__device__ __forceinline__ bool sched_read_mma(SS& sb, int e, int4& ent, volatile int* abort, uint64_t limit_ns) {
-  const int slot = e % kSchedSlots;
-  if (!mbar_wait(&sb.sched_full[kMmaRing][slot], (e / kSchedSlots) & 1, abort, limit_ns)) return false;
-  ent = sb.sched[kMmaRing][slot];
-  mbar_arrive(&sb.sched_empty[kMmaRing][slot]);
-  return true;
 }
 
 // --------------------------------------------------------------- MMA issuers
@@ -285,11 +284,18 @@ __device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* q_stage,
   int j = 0, nq = 0;
   bool ok = true;
   for (;;) {
-    int4 ent;
-    if (!sched_read_mma(sb, j, ent, abort, p.wait_ns)) {
+    const int slot = j % RK;
+    // K(j) has landed, and with it tile j's entry of the MMA ring (written
+    // before K(j) was loaded; the end marker completes the barrier without a
+    // copy); S(j) overwrites S(j-1), so its softmax warpgroup must have read
+    // it.  Both are probed together.
+    if (!mbar_wait_both(&sb.k_full[slot], (j / RK) & 1, &sb.s_free[(j - 1) & 1], ((j - 1) >> 1) & 1, j >= 1,
+                        abort, p.wait_ns)) {
       ok = false;
       break;
     }
+    const int4 ent = sb.sched[kMmaRing][j % kSchedSlots];
+    mbar_arrive(&sb.sched_empty[kMmaRing][j % kSchedSlots]);
     if (ent.z & kEntEnd) break;
     if (ent.z & kEntFirst) {
       // Q in TMEM was last read by the S products of unit nq - 1.
@@ -309,16 +315,6 @@ __device__ void attn_mma_s(const AttnParams& p, uint32_t tmem, uint8_t* q_stage,
                          smem_desc_sw128(q_base + (kk >> 2) * (128 * 128) + (kk & 3) * 32, 16, 1024));
       umma_commit(&sb.q_stage_free);
       ++nq;
-    }
-    const int slot = j % RK;
-    if (!mbar_wait(&sb.k_full[slot], (j / RK) & 1, abort, p.wait_ns)) {
-      ok = false;
-      break;
-    }
-    // S(j) overwrites S(j-1): its softmax warpgroup must have read it.
-    if (j >= 1 && !mbar_wait(&sb.s_free[(j - 1) & 1], ((j - 1) >> 1) & 1, abort, p.wait_ns)) {
-      ok = false;
-      break;
     }
     tc_fence_after_sync();
     const uint32_t s_col = C::kTmemS;
@@ -353,11 +349,16 @@ __device__ void attn_mma_pv(const AttnParams& p, uint32_t tmem, uint8_t* ring,
   int j = 0, nu = 0;
   bool ok = true;
   for (;;) {
-    int4 ent;
-    if (!sched_read_mma(sb, j, ent, abort, p.wait_ns)) {
+    const int slot = j % RV;
+    // V(j) has landed, and with it tile j's entry of the MMA ring (written
+    // before V(j) was loaded; the end marker completes the barrier without a
+    // copy).
+    if (!mbar_wait(&sb.v_full[slot], (j / RV) & 1, abort, p.wait_ns)) {
       ok = false;
       break;
     }
+    const int4 ent = sb.sched[kMmaRing][j % kSchedSlots];
+    mbar_arrive(&sb.sched_empty[kMmaRing][j % kSchedSlots]);
     if (ent.z & kEntEnd) break;
     const bool first = (ent.z & kEntFirst) != 0;
     if (first) {
@@ -369,12 +370,7 @@ __device__ void attn_mma_pv(const AttnParams& p, uint32_t tmem, uint8_t* ring,
       }
       ++nu;
     }
-    const int slot = j % RV;
     if (!mbar_wait(&sb.p_full[j & 1], (j >> 1) & 1, abort, p.wait_ns)) {
-      ok = false;
-      break;
-    }
-    if (!mbar_wait(&sb.v_full[slot], (j / RV) & 1, abort, p.wait_ns)) {
       ok = false;
       break;
     }

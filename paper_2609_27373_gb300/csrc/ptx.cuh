@@ -78,6 +78,10 @@ __device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
   return done != 0;
 }
 
+// Limits below this are checked on every poll (a deliberately short limit,
+// set to exercise the timeout path); longer ones every few polls.
+constexpr uint64_t kShortWaitNs = 1000000ull;
+
 // Waits for the phase with the given parity to complete.  Returns false if
 // *abort becomes non-zero or the wait exceeds limit_ns (kWaitLimitNs unless
 // the launch chose a shorter limit); never spins forever.
@@ -87,7 +91,27 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
   const uint64_t t0 = global_timer_ns();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 31u) == 0) {
+    if ((it & 31u) == 0 || limit_ns < kShortWaitNs) {
+      if (*abort) return false;
+      if (global_timer_ns() - t0 > limit_ns) return false;
+    }
+  }
+}
+
+// Waits for two phases at once (the second only if need_b), probing both on
+// every pass without suspending, so that the two probe latencies overlap.
+// Bounded like mbar_wait.
+__device__ __forceinline__ bool mbar_wait_both(uint64_t* a, uint32_t parity_a, uint64_t* b, uint32_t parity_b,
+                                               bool need_b, volatile int* abort, uint64_t limit_ns = kWaitLimitNs) {
+  bool da = mbar_test_wait(a, parity_a);
+  bool db = need_b ? mbar_test_wait(b, parity_b) : true;
+  if (da && db) return true;
+  const uint64_t t0 = global_timer_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (!da) da = mbar_test_wait(a, parity_a);
+    if (!db) db = mbar_test_wait(b, parity_b);
+    if (da && db) return true;
+    if ((it & 255u) == 0 || limit_ns < kShortWaitNs) {
       if (*abort) return false;
       if (global_timer_ns() - t0 > limit_ns) return false;
     }
