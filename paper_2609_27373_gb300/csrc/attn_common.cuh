@@ -118,6 +118,26 @@ __device__ __forceinline__ float exp2_scaled_groups(float (&s)[N], float scale, 
   return total;
 }
 
+// Column sums over the 32 lanes of a warp: v[i] holds this lane's value of
+// column i; returns the sum of column `lane`.  Each step exchanges half of
+// the remaining columns with the lane `o` away (o = 16, 8, 4, 2, 1), 31
+// shuffles in all.  The additions pair the lanes exactly as a butterfly
+// reduction with the same offsets does, so every column sum is the same bit
+// for bit.
+__device__ __forceinline__ float warp_column_sums(float (&v)[32], int lane) {
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) {
+    const bool upper = (lane & o) != 0;
+#pragma unroll
+    for (int i = 0; i < o; ++i) {
+      const float send = upper ? v[i] : v[i + o];
+      const float keep = upper ? v[i + o] : v[i];
+      v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+    }
+  }
+  return v[0];
+}
+
 // Key tiles of one unit in ascending order, with their sub-block masks
 // (S = 128 / BLK).  Dense: tiles 0..last, every sub-block (the causal limit is
 // applied per row).  Sparse: the merge of the support lists of the unit's S

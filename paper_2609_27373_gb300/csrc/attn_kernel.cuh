@@ -582,13 +582,19 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
       // Dense variants: tile t of the unit is key tile t, holding key blocks
       // t * S .. t * S + S - 1.
       const int n_kb = min(ei.n_kt * S, p.n_blocks);
-      for (int kb = 0; kb < n_kb; ++kb) {
-        const int t = kb / S;
-        const float lc = *lc_at((ei.j0 + t) & 1, ei.nu, t, kb - t * S);
-        float v = (row < p.seqlen) ? ex2_approx(lc - lse) : 0.0f;
+      // 32 key blocks per pass: their partials are loaded together, and the
+      // warp's 32 column sums end one per lane.
+      for (int kb0 = 0; kb0 < n_kb; kb0 += 32) {
+        float v[32];
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-        if (lane == 0) ws[wq * p.n_blocks + kb] = v;
+        for (int i = 0; i < 32; ++i) {
+          const int kb = kb0 + i, t = kb / S;
+          v[i] = (kb < n_kb) ? *lc_at((ei.j0 + t) & 1, ei.nu, t, kb - t * S) : -INFINITY;
+        }
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = (row < p.seqlen) ? ex2_approx(v[i] - lse) : 0.0f;
+        const float sum = warp_column_sums(v, lane);
+        if (kb0 + lane < n_kb) ws[wq * p.n_blocks + kb0 + lane] = sum;
       }
       // Orders the four warps' writes before the reads below (release /
       // acquire at CTA scope).
