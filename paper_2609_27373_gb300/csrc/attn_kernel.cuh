@@ -549,15 +549,19 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     const int row = qt * 128 + r;
     const float inv_l = l_row > 0.0f ? 1.0f / l_row : 0.0f;
     // O / l through this warp's staging box (32 rows x 64 columns, 128-byte
-    // swizzle) and a TMA store per 64 columns; rows past seqlen are dropped.
-    // The other warpgroup's stores from the box were read before its
-    // publication (above).
+    // swizzle): each thread writes its row, then the warp reads the box back
+    // four rows at a time (eight lanes per 128-byte row segment) and stores
+    // it to global memory, so that each store instruction covers whole
+    // segments.  Rows past seqlen and columns past D are dropped.  (TMA
+    // stores from the box queue behind the K/V loads in the copy engine and
+    // the box could not be refilled until they had read it.)  The epilogues
+    // of consecutive units never overlap: L of a unit waits for the other
+    // warpgroup's publication, which that warpgroup makes after any
+    // epilogue of its own.
     uint8_t* stage = out_stage + wq * (32 * 128);
+    __nv_bfloat16* o_rows = p.O + ((size_t)(b * p.n_heads + h) * p.seqlen + qt * 128 + wq * 32) * D;
 #pragma unroll
     for (int hb = 0; hb < C::kBoxes; ++hb) {
-      // The previous store from the staging box has read it.
-      if (lane == 0) tma_store_wait_read();
-      __syncwarp();
 #pragma unroll
       for (int c = 0; c < 8; ++c) {
         const int col = hb * 64 + c * 8;
@@ -567,12 +571,16 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
           q[e] = (col + 2 * e + 1 < D) ? pack_bf16x2(o[col + 2 * e] * inv_l, o[col + 2 * e + 1] * inv_l) : 0u;
         st_shared_v4(smem_u32(stage + lane * 128 + ((c ^ (lane & 7)) << 4)), q[0], q[1], q[2], q[3]);
       }
-      fence_proxy_async_smem();
       __syncwarp();
-      if (lane == 0) {
-        tma_store_3d(mapO, stage, hb * 64, qt * 128 + wq * 32, b * p.n_heads + h);
-        tma_store_commit();
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int rr = i * 4 + (lane >> 3), c = lane & 7;
+        const uint4 val = ld_shared_v4(smem_u32(stage + rr * 128 + ((c ^ (rr & 7)) << 4)));
+        const int col = hb * 64 + c * 8;
+        if (qt * 128 + wq * 32 + rr < p.seqlen && col < D)
+          *reinterpret_cast<uint4*>(o_rows + (size_t)rr * D + col) = val;
       }
+      __syncwarp();
     }
     if constexpr (MODE == kDenseMass) {
       // Block mass (Eq. 5): per row 2^(lc - lse), summed over the rows of
@@ -630,11 +638,6 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     if (n_pub >= 1 && !warp_wait(&sb.l_ack[w], (n_pub - 1) & 1, abort, p.wait_ns)) return false;
     sb.lx[w][r] = fresh ? 0.0f : l_w;
     sb.lm[w][r] = fresh ? -INFINITY : m_w;
-    // The staging boxes are shared by the two warpgroups and a bulk-group
-    // wait covers only this thread's stores: before L (which waits for this
-    // publication) writes box wq, this warp's earlier stores from it must
-    // have read it.
-    if (lane == 0) tma_store_wait_read();
     __syncwarp();
     if (lane == 0) mbar_arrive(&sb.l_pub[w]);
     ++n_pub;
