@@ -283,14 +283,13 @@ __device__ __forceinline__ void tmem_load_row(uint32_t addr, float (&x)[N]) {
   }
 }
 
-// Loads this thread's row of an S tile (kTileN columns) and applies the
-// causal / support masks: column c of key sub-block k = c / BLK is kept if
+// Applies the causal / support masks to this thread's row of an S tile
+// (kTileN columns): column c of key sub-block k = c / BLK is kept if
 // bit k of `sub` is set and c <= lim (keys with c > lim are in the future of
 // this row).
 template <int BLK>
-__device__ __forceinline__ void load_s_row(uint32_t addr, float (&s)[kTileN], uint32_t sub, int lim) {
+__device__ __forceinline__ void mask_s_row(float (&s)[kTileN], uint32_t sub, int lim) {
   constexpr int S = kTileN / BLK;
-  tmem_load_row<kTileN>(addr, s);
   if (sub != (1u << S) - 1u || lim < kTileN - 1) {
     // Per sub-block limit: lim where the row attends the sub-block, else the
     // column before it, so that a single compare masks the column.
@@ -300,6 +299,13 @@ __device__ __forceinline__ void load_s_row(uint32_t addr, float (&s)[kTileN], ui
 #pragma unroll
     for (int c = 0; c < kTileN; ++c) s[c] = (c > lim_k[c / BLK]) ? -INFINITY : s[c];
   }
+}
+
+// Loads this thread's row of an S tile and applies the masks.
+template <int BLK>
+__device__ __forceinline__ void load_s_row(uint32_t addr, float (&s)[kTileN], uint32_t sub, int lim) {
+  tmem_load_row<kTileN>(addr, s);
+  mask_s_row<BLK>(s, sub, lim);
 }
 
 }  // namespace wise

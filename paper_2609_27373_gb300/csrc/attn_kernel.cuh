@@ -444,11 +444,13 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     const uint32_t sub = ((uint32_t)key >> (16 + qsub * S)) & ((1u << S) - 1u);
     const int lim = cur_row - kb * kTileN;  // keys kb*128 + c with c > lim are in the future
     float s[kTileN];
-    load_s_row<BLK>(lane_tmem + s_col, s, sub, lim);
-    // S(j) is in registers: S(j+1) may overwrite it.
+    tmem_load_row<kTileN>(lane_tmem + s_col, s);
+    // S(j) is in registers: S(j+1) may overwrite it (released before the
+    // masks, which are on the path of the next S product otherwise).
     tc_fence_before_sync();
     __syncwarp();
     if (lane == 0) mbar_arrive(&sb.s_free[w]);
+    mask_s_row<BLK>(s, sub, lim);
     const float m_tile = row_max(s) * p.scale_log2;
     // Running max after the previous tile (the other warpgroup's).
     float m_prev = -INFINITY;
