@@ -88,7 +88,7 @@ struct AttnCfg {
   static constexpr int kQBytes = kBoxes * 128 * 128;    // one 128-row Q tile (staging)
   static constexpr int kKVBytes = kBoxes * kTileN * 128; // one 128-row K or V tile (one ring entry)
   // Static shared memory (barriers, schedule ring, row exchange buffers).
-  static constexpr int kStaticReserve = 7 * 1024;
+  static constexpr int kStaticReserve = 10 * 1024;
   // Dynamic shared memory available after the 1024-byte alignment slack.
   static constexpr int kBudget = 227 * 1024 - 1024 - kStaticReserve;
   // Epilogue staging: per softmax warp of L, 32 rows x 64 columns of O
@@ -108,8 +108,9 @@ struct AttnCfg {
   static constexpr uint32_t kTmemPCols = 64;
   static constexpr uint32_t kTmemO = 384;     // O accumulator
   static constexpr uint32_t kTmemCols = 512;
-  // Warps 0-7 softmax, 8 producer, 9 and 10 MMA issuers, 11 idle (it
-  // completes warpgroup 2 for setmaxnreg).  Launch: 384 x 168 registers;
+  // Warps 0-7 softmax, 8 producer, 9 and 10 MMA issuers, 11 schedule
+  // stager (sparse with blocks of 32 or 64; otherwise idle, it completes
+  // warpgroup 2 for setmaxnreg).  Launch: 384 x 168 registers;
   // after the split 256 x kRegsSoftmax + 128 x kRegsOther = 64512.
   static constexpr int kThreads = 384;
   static constexpr int kRegsSoftmax = 216;
@@ -121,6 +122,22 @@ struct AttnCfg {
   static_assert(D <= 128, "TMEM budget");
   static_assert(256 * kRegsSoftmax + 128 * kRegsOther <= kThreads * 168, "register split");
 };
+
+// Sparse tile schedules staged by warp 11 (blocks of 32 and 64, S > 1 lists
+// per unit): entries per slot (a unit's tiles, as schedule keys), the key
+// tiles a staged unit may span, and the slots.  A launch stages when every
+// unit fits: cap * S <= kStageKeys (each accepted list entry adds at most one
+// tile) and n_qtiles <= kStageTiles.  With one list per unit (block 128) the
+// producer's own merge measured faster than staging (4K late step 68.5
+// against 74 us).
+constexpr int kStageKeys = 128;
+constexpr int kStageTiles = 256;
+constexpr int kStageSlots = 4;
+template <int BLK, int MODE>
+__device__ __forceinline__ bool sched_staging(const AttnParams& p) {
+  constexpr int S = kTileN / BLK;
+  return MODE == kSparse && S > 1 && p.cap <= kStageKeys / S && p.n_qtiles <= kStageTiles;
+}
 
 template <int RK, int RV>
 struct SharedState {
@@ -149,9 +166,113 @@ struct SharedState {
   float mx[2][2][128];   // [warpgroup][slot][row] running max after a tile
   float lx[2][128];      // [warpgroup][row] E's row-sum part at the end of a unit
   float lm[2][128];      // [warpgroup][row] the max that part refers to
+  // Staged tile schedules (slot = the unit's position in the CTA's sequence
+  // mod kStageSlots): the keys of the unit's tiles and their number n (-1 - n when a
+  // count or a list entry of the unit was invalid).
+  uint64_t list_full[kStageSlots];   // staged (warp 11)
+  uint64_t list_empty[kStageSlots];  // the producer has read the slot
+  int32_t stage_keys[kStageSlots][kStageKeys];
+  int32_t stage_n[kStageSlots];
+  uint32_t stage_tmask[kStageTiles];  // warp 11 scratch: mask of each key tile
   uint32_t tmem_base;
   int abort;
 };
+
+// -------------------------------------------------------- schedule stager
+// Sparse launches that stage (sched_staging): warp 11 walks the CTA's units
+// in the producer's order, at most kStageSlots units ahead, and turns each unit's S
+// support lists into its tile schedule in shared memory, with the 32 lanes
+// working together: an entry of list q is accepted if it lies in [0, q0 + q]
+// and exceeds every accepted entry before it in its list (= every in-range
+// entry before it: an in-range entry that was not accepted lies below an
+// accepted one), which a prefix max over the list finds; the accepted key
+// blocks are OR-ed into a mask per key tile; the tiles with a non-empty mask
+// are compacted in ascending order.  The producer then reads a unit's keys
+// from shared memory instead of merging the lists itself, one dependent
+// global load per list entry on a thread that shares its scheduler with two
+// busy softmax warps.
+template <int D, int BLK, int MODE>
+__device__ void attn_sched_stager(const AttnParams& p, SharedState<AttnCfg<D>::kRingK, AttnCfg<D>::kRingV>& sb) {
+  constexpr int S = kTileN / BLK;
+  constexpr int kCap = kStageKeys / S;      // list positions staged per query block (>= cap)
+  constexpr int kRegs = kStageKeys / 32;    // entry e = lane + 32 i in register i
+  constexpr int kRegsPerList = kCap / 32;   // list q: registers q * kRegsPerList ..
+  const int lane = threadIdx.x & 31;
+  volatile int* abort = &sb.abort;
+  const int G = gridDim.x, c = blockIdx.x;
+  int n_st = 0;
+  bool ok = true;
+  for (int k = 0; ok && k * G < p.n_units; ++k) {
+    const int u = k * G + ((k & 1) ? G - 1 - c : c);
+    if (u >= p.n_units) continue;
+    int b, h, qt;
+    decode_unit(p, u, b, h, qt);
+    const int q0 = qt * S;
+    const size_t row0 = ((size_t)b * p.n_kv_heads + h / p.group) * p.n_blocks + q0;
+    const int slot = n_st % kStageSlots;
+    // The producer has read the schedule that used the slot before.
+    if (n_st >= kStageSlots && !warp_wait(&sb.list_empty[slot], ((n_st / kStageSlots) - 1) & 1, abort, p.wait_ns)) {
+      ok = false;
+      break;
+    }
+    int bad = 0;
+    int cnt[S];
+#pragma unroll
+    for (int q = 0; q < S; ++q) cnt[q] = (q0 + q < p.n_blocks) ? __ldg(p.counts + row0 + q) : 0;
+    // The entries are loaded alongside the counts (every position below cap
+    // exists), so that the unit costs one memory latency.
+    int v[kRegs];
+    bool live[kRegs], acc[kRegs];
+#pragma unroll
+    for (int i = 0; i < kRegs; ++i) {
+      const int q = i / kRegsPerList, x = (i % kRegsPerList) * 32 + lane;
+      v[i] = (q0 + q < p.n_blocks && x < p.cap) ? __ldg(p.idx + (row0 + q) * p.cap + x) : -1;
+    }
+#pragma unroll
+    for (int q = 0; q < S; ++q) cnt[q] = (q0 + q < p.n_blocks) ? clamp_count(cnt[q], p.cap, bad) : 0;
+#pragma unroll
+    for (int i = 0; i < kRegs; ++i) live[i] = (i % kRegsPerList) * 32 + lane < cnt[i / kRegsPerList];
+    int carry = -1;  // max of the in-range entries of the list's earlier registers
+#pragma unroll
+    for (int i = 0; i < kRegs; ++i) {
+      const int q = i / kRegsPerList;
+      if (i % kRegsPerList == 0) carry = -1;
+      const bool in_range = live[i] && v[i] >= 0 && v[i] <= q0 + q;
+      int m = in_range ? v[i] : -1;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int t = __shfl_up_sync(0xffffffffu, m, o);
+        if (lane >= o) m = max(m, t);
+      }
+      int before = __shfl_up_sync(0xffffffffu, m, 1);
+      before = max(lane == 0 ? -1 : before, carry);
+      acc[i] = in_range && v[i] > before;
+      if (live[i] && !acc[i]) bad = 1;
+      carry = max(carry, __shfl_sync(0xffffffffu, m, 31));
+    }
+    // Masks of the key tiles 0..qt (every accepted block lies in one).
+    for (int t = lane; t <= qt; t += 32) sb.stage_tmask[t] = 0u;
+    __syncwarp();
+#pragma unroll
+    for (int i = 0; i < kRegs; ++i)
+      if (acc[i]) atomicOr(&sb.stage_tmask[v[i] / S], 1u << ((i / kRegsPerList) * S + v[i] % S));
+    __syncwarp();
+    int n = 0;
+    for (int t0 = 0; t0 <= qt; t0 += 32) {
+      const int t = t0 + lane;
+      const uint32_t m = t <= qt ? sb.stage_tmask[t] : 0u;
+      const uint32_t bal = __ballot_sync(0xffffffffu, m != 0u);
+      if (m) sb.stage_keys[slot][n + __popc(bal & ((1u << lane) - 1u))] = (int)((uint32_t)t | (m << 16));
+      n += __popc(bal);
+    }
+    bad = __any_sync(0xffffffffu, bad);
+    if (lane == 0) sb.stage_n[slot] = bad ? -1 - n : n;
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&sb.list_full[slot]);
+    ++n_st;
+  }
+  if (!ok) raise_status(p, &sb.abort, kStatusTimeout);
+}
 
 // ------------------------------------------------------------------ producer
 template <int D, int BLK, int MODE>
@@ -165,6 +286,8 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
   volatile int* abort = &sb.abort;
   int jk = 0, jv = 0, nq = 0, bad = 0;
   int jt = 0, n_empty = 0;  // tiles and units without tiles scheduled so far
+  int n_units = 0;          // units walked so far
+  const bool staged = sched_staging<BLK, MODE>(p);
   bool ok = true;
   // Writes the next entry of a ring.  Its position follows from the counts:
   // the MMA ring holds every tile, ring 1 the odd tiles, ring 0 the even
@@ -199,10 +322,36 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
     decode_unit(p, u, b, h, qt);
     const int kvh = h / p.group;
     const int z = b * p.n_kv_heads + kvh;
-    auto it = make_iter<BLK, MODE>(p, b, kvh, qt);
+    // The unit's tiles: from warp 11's staged schedule, or merged here.
+    const int lslot = n_units % kStageSlots;
+    int st_n = 0, st_t = 0;
+    TileIter<BLK, MODE> it;
+    if (staged) {
+      if (!mbar_wait(&sb.list_full[lslot], (n_units / kStageSlots) & 1, abort, p.wait_ns)) {
+        ok = false;
+        break;
+      }
+      st_n = sb.stage_n[lslot];
+      if (st_n < 0) {
+        bad = 1;
+        st_n = -1 - st_n;
+      }
+    } else {
+      it = make_iter<BLK, MODE>(p, b, kvh, qt);
+    }
+    auto next_tile = [&](int& kt, uint32_t& m) -> bool {
+      if (staged) {
+        if (st_t >= st_n) return false;
+        const int key = sb.stage_keys[lslot][st_t++];
+        kt = key & 0xFFFF;
+        m = (uint32_t)key >> 16;
+        return true;
+      }
+      return it.next(kt, m);
+    };
     int kb;
     uint32_t mask;
-    bool have = it.next(kb, mask);
+    bool have = next_tile(kb, mask);
     if (!have) {
       if (!emit(0, 0, u, kEntEmpty, 0)) ok = false;
       ++n_empty;
@@ -212,7 +361,7 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
     for (int t = 0; have && ok; ++t) {
       int nkb;
       uint32_t nmask;
-      const bool more = it.next(nkb, nmask);
+      const bool more = next_tile(nkb, nmask);
       const int flags = (first ? kEntFirst : 0) | (more ? 0 : kEntLast) | (unit_ix << kEntUnitShift);
       const int key = (int)((uint32_t)kb | (mask << 16));
       if (!emit(kMmaRing, key, u, flags, t) || !emit(jt & 1, key, u, flags, t)) {
@@ -247,7 +396,12 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
       have = more;
       first = false;
     }
-    bad |= it.bad;
+    if (staged) {
+      mbar_arrive(&sb.list_empty[lslot]);  // the schedule has been read
+    } else {
+      bad |= it.bad;
+    }
+    ++n_units;
   }
   if (ok && have_prev && !load(mapV, v_ring, sb.v_full, sb.v_empty, RV, jv, prev_kb, prev_z)) ok = false;
   for (int rw = 0; rw < 3 && ok; ++rw)
@@ -763,6 +917,10 @@ __global__ void __launch_bounds__(AttnCfg<D>::kThreads, 1)
       mbar_init(&sb.o_full[b], 1);
     }
     mbar_init(&sb.o_free, 4);
+    for (int b = 0; b < kStageSlots; ++b) {
+      mbar_init(&sb.list_full[b], 1);
+      mbar_init(&sb.list_empty[b], 1);
+    }
     mbar_init(&sb.s_done, 1);
     mbar_init(&sb.pv_done, 1);
     fence_mbar_init();
@@ -793,6 +951,8 @@ __global__ void __launch_bounds__(AttnCfg<D>::kThreads, 1)
       if (lane == 0) attn_mma_s<D, BLK, MODE>(p, tmem, q_stage, ring, sb);
     } else if (warp == C::kMmaPVWarp) {
       if (lane == 0) attn_mma_pv<D, BLK, MODE>(p, tmem, ring, sb);
+    } else if (sched_staging<BLK, MODE>(p)) {
+      attn_sched_stager<D, BLK, MODE>(p, sb);  // warp 11
     }
   }
 
