@@ -202,6 +202,35 @@ def test_inconsistent_support_is_skipped_and_flagged(name):
     assert_close_o(bf16_dev_to_f64(O), want)
 
 
+@pytest.mark.parametrize("name", ["d128_b32", "d64_b32_gqa_ragged", "d64_b64_ragged", "d128_b64_gqa"])
+def test_staged_and_merged_schedules_agree(name):
+    """Blocks 32 and 64 take their tile schedules from the staging warp while
+    cap * (128 / B) <= 128, else from the producer's own merge of the lists.
+    The same support, stored once at the largest staged cap and once with one
+    more (empty) column, must give the same output bits, valid or not."""
+    shape, Q, K, V = _inputs(name)
+    nb, S = shape.n_blocks, 128 // shape.block
+    cap = 128 // S
+    idx, counts = synth.random_support(shape.batch, shape.n_kv_heads, nb, cap, seed=7, density=0.6)
+    # one malformed row (unordered, duplicate, out of range) in both layouts
+    q = min(5, nb - 1)
+    idx[0, 0, q, :4] = [q, 0, 0, nb + 3]
+    counts[0, 0, q] = 4
+    wide = np.full(idx.shape[:-1] + (cap + 1,), -1, dtype=np.int32)
+    wide[..., :cap] = idx
+    O_staged = _sparse(shape, Q, K, V, idx, counts)
+    st_staged = wise.wise_get_status()
+    O_merged = _sparse(shape, Q, K, V, wide, counts)
+    st_merged = wise.wise_get_status()
+    assert st_staged == st_merged == wise.WISE_ERR_BAD_SUPPORT
+    assert torch.equal(O_staged.view(torch.int16), O_merged.view(torch.int16))
+    fixed_idx, fixed_counts = idx.copy(), counts.copy()
+    fixed_idx[0, 0, q, :4] = [q, -1, -1, -1]
+    fixed_counts[0, 0, q] = 1
+    want = orc.sparse_attention(Q, K, V, fixed_idx, fixed_counts, shape.block)
+    assert_close_o(bf16_dev_to_f64(O_staged), want)
+
+
 def test_tiny_workload_trajectory_end_to_end():
     """The tiny workload (L=512, 4 heads, d=64, block 64): 3 discovery steps,
     one selection, 5 late steps, through the WiseAttention driver."""
