@@ -10,9 +10,11 @@ timed region starts.
 
 Reported (one JSON line on rank 0):
   value            late-step attention ms per recurrent step (sparse kernel,
-                   CUDA events on the launching stream, mean over late steps)
+                   CUDA events on the launching stream around the late steps
+                   after the first, which run back to back as in the
+                   trajectory, divided by their number; mean over trajectories)
   dense_ms         the library's own dense kernel (no mass) on the same late
-                   inputs; speedup = dense_ms / value
+                   inputs, timed the same way; speedup = dense_ms / value
   roofline         the sparse kernel's algorithmic tensor FLOPs per launch
                    over its mean launch time, against the measured bf16 peak
   e2e              the same late step through the C ABI with Q/K/V copied from
@@ -313,15 +315,34 @@ def main():
     layer = wise.WiseAttention(shape, sel, wl.n_discovery)
     stream = torch.cuda.current_stream()
 
+    def per_call_ms(calls):
+        """Mean time per call of `calls` run back to back on the stream between
+        one pair of CUDA events.  Consecutive attention launches overlap their
+        set-up with the end of the previous one (programmatic dependent
+        launch), as they do in a trajectory; an event recorded between two
+        launches would keep them apart."""
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for c in calls:
+            c()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / len(calls)
+
     def trajectory(ev=None):
+        """One trajectory.  With `ev`: events around each discovery step and the
+        first late step (it also runs the selection), then one pair around the
+        remaining late steps, which run back to back."""
         layer.selected = False
         for t in range(wl.steps):
             Q, K, V = dev_steps[t]
-            if ev is not None:
+            if ev is not None and t <= wl.n_discovery + 1:
                 ev[t][0].record(stream)
             layer.step(t, Q, K, V, O)
-            if ev is not None:
+            if ev is not None and t <= wl.n_discovery:
                 ev[t][1].record(stream)
+        if ev is not None:
+            ev[wl.n_discovery + 1][1].record(stream)
 
     for _ in range(args.warmup):
         trajectory()
@@ -349,14 +370,11 @@ def main():
     total_ms = t_start.elapsed_time(t_end)
     disc_ms, sel_ms, late_ms = [], [], []
     for k in range(args.steps):
-        for t in range(wl.steps):
-            ms = evs[k][t][0].elapsed_time(evs[k][t][1])
-            if t < wl.n_discovery:
-                disc_ms.append(ms)
-            elif t == wl.n_discovery:
-                late_ms.append(ms)  # includes the selection launch; split below
-            else:
-                late_ms.append(ms)
+        for t in range(wl.n_discovery):
+            disc_ms.append(evs[k][t][0].elapsed_time(evs[k][t][1]))
+        # the late steps after the first, back to back (the first also ran the
+        # selection: timed alone below)
+        late_ms.append(evs[k][wl.n_discovery + 1][0].elapsed_time(evs[k][wl.n_discovery + 1][1]) / (n_late - 1))
     # the first late step also ran the selection; time the selection alone
     sel_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     for k in range(args.steps):
@@ -365,19 +383,12 @@ def main():
         sel_ev[k][1].record(stream)
     torch.cuda.synchronize()
     sel_ms = [a.elapsed_time(b) for a, b in sel_ev]
-    late_only = [late_ms[i] for i in range(len(late_ms)) if i % n_late != 0]  # steps without the selection
+    late_only = late_ms  # late steps without the selection
 
     # ---- own dense kernel on the same late inputs
-    dense_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_late)]
-    dense_ms = []
-    for k in range(max(1, args.steps // 2)):
-        for i, t in enumerate(range(wl.n_discovery, wl.steps)):
-            Q, K, V = dev_steps[t]
-            dense_ev[i][0].record(stream)
-            wise.wise_full_attn_accumulate(shape, Q, K, V, O)
-            dense_ev[i][1].record(stream)
-        torch.cuda.synchronize()
-        dense_ms += [a.elapsed_time(b) for a, b in dense_ev]
+    dense_calls = [lambda t=t: wise.wise_full_attn_accumulate(shape, *dev_steps[t], O)
+                   for t in range(wl.n_discovery, wl.steps)]
+    dense_ms = [per_call_ms(dense_calls) for _ in range(max(1, args.steps // 2))]
 
     # ---- end to end through host buffers (pinned), late steps
     pinned = [tuple(torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).pin_memory() for x in host_steps[t])
@@ -430,14 +441,8 @@ def main():
     nb = shape.n_blocks
     all_idx, all_counts = synth.all_blocks_support(wl.batch, wl.n_kv_heads, nb)
     all_idx, all_counts = torch.from_numpy(all_idx).cuda(), torch.from_numpy(all_counts).cuda()
-    ab_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_late)]
-    for i, t in enumerate(range(wl.n_discovery, wl.steps)):
-        Q, K, V = dev_steps[t]
-        ab_ev[i][0].record(stream)
-        wise.wise_sparse_attn(shape, Q, K, V, all_idx, all_counts, O)
-        ab_ev[i][1].record(stream)
-    torch.cuda.synchronize()
-    all_blocks_ms = statistics.mean(a.elapsed_time(b) for a, b in ab_ev)
+    all_blocks_ms = per_call_ms([lambda t=t: wise.wise_sparse_attn(shape, *dev_steps[t], all_idx, all_counts, O)
+                                 for t in range(wl.n_discovery, wl.steps)])
 
     # ---- routing diagnostic: share of each late step's full attention kept
     # by the frozen support (the step's own block mass, then the support sum)
@@ -476,15 +481,11 @@ def main():
             wise.wise_full_attn_accumulate(shape, *dev_steps[t], O, diag_mass, 0)
             wise.wise_support_mass(shape, diag_mass, ws_idx[k], ws_cnt[k], retained)
             rm.append(float(retained.mean()))
-        evs_k = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_late)]
-        for i, t in enumerate(range(wl.n_discovery, wl.steps)):
-            evs_k[i][0].record(stream)
-            wise.wise_sparse_attn(shape, *dev_steps[t], ws_idx[k], ws_cnt[k], O)
-            evs_k[i][1].record(stream)
-        torch.cuda.synchronize()
+        sp_k = per_call_ms([lambda t=t, k=k: wise.wise_sparse_attn(shape, *dev_steps[t], ws_idx[k], ws_cnt[k], O)
+                            for t in range(wl.n_discovery, wl.steps)])
         supports[k] = {"density": round(float(ws_cnt[k].sum()) / admissible, 4),
                        "retained_mass": round(statistics.mean(rm), 4),
-                       "sparse_ms": round(statistics.mean(a.elapsed_time(b) for a, b in evs_k), 5)}
+                       "sparse_ms": round(sp_k, 5)}
 
     # ---- stability of the rolling working set at the discovery endpoint
     # (appendix "Stability of the Deployed Working Set"): W(t) = union of the
@@ -502,14 +503,10 @@ def main():
 
     # ---- Freeze-A control: the selected support with the within-support
     # distribution of the last discovery step, applied to each late step's V
-    fz_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_late)]
     Q_td, K_td, _ = dev_steps[wl.n_discovery - 1]
-    for i, t in enumerate(range(wl.n_discovery, wl.steps)):
-        fz_ev[i][0].record(stream)
-        wise.wise_freeze_a_attn(shape, Q_td, K_td, dev_steps[t][2], layer.idx, layer.counts, O)
-        fz_ev[i][1].record(stream)
-    torch.cuda.synchronize()
-    freeze_a_ms = statistics.mean(a.elapsed_time(b) for a, b in fz_ev)
+    freeze_a_ms = per_call_ms([lambda t=t: wise.wise_freeze_a_attn(shape, Q_td, K_td, dev_steps[t][2], layer.idx,
+                                                                   layer.counts, O)
+                               for t in range(wl.n_discovery, wl.steps)])
 
     # ---- Freeze-A with the distribution stored once (row-max-relative bf16
     # tiles + 1/sum per row) and a block-sparse P V product per late step:
@@ -523,13 +520,10 @@ def main():
     pr_ev[0].record(stream)
     wise.wise_freeze_a_probs(shape, Q_td, K_td, layer.idx, layer.counts, P_frz, inv_l)
     pr_ev[1].record(stream)
-    for rep in range(2):  # the first pass warms up
-        for i, t in enumerate(range(wl.n_discovery, wl.steps)):
-            fz_ev[i][0].record(stream)
-            wise.wise_frozen_pv(shape, P_frz, inv_l, dev_steps[t][2], layer.idx, layer.counts, O)
-            fz_ev[i][1].record(stream)
-        torch.cuda.synchronize()
-    frozen_pv_ms = statistics.mean(a.elapsed_time(b) for a, b in fz_ev)
+    pv_calls = [lambda t=t: wise.wise_frozen_pv(shape, P_frz, inv_l, dev_steps[t][2], layer.idx, layer.counts, O)
+                for t in range(wl.n_discovery, wl.steps)]
+    per_call_ms(pv_calls)  # warm-up
+    frozen_pv_ms = per_call_ms(pv_calls)
     # Algorithmic bytes per launch: the stored tiles of every walk, V once
     # (every key block is selected by some query tile of its head), O, inv_l.
     walk_tiles = 0
@@ -564,14 +558,10 @@ def main():
     O32 = torch.empty_like(steps32[0][0])
     for t in range(wl32.n_discovery + 1):
         layer32.step(t, *steps32[t], O32)
-    ev32 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(late32)]
-    for rep in range(2):  # the first pass warms up
-        for i, t in enumerate(range(wl32.n_discovery, wl32.n_discovery + late32)):
-            ev32[i][0].record(stream)
-            wise.wise_sparse_attn(shape32, *steps32[t], layer32.idx, layer32.counts, O32)
-            ev32[i][1].record(stream)
-        torch.cuda.synchronize()
-    b32_ms = statistics.mean(a.elapsed_time(b) for a, b in ev32)
+    calls32 = [lambda t=t: wise.wise_sparse_attn(shape32, *steps32[t], layer32.idx, layer32.counts, O32)
+               for t in range(wl32.n_discovery, wl32.n_discovery + late32)]
+    per_call_ms(calls32)  # warm-up
+    b32_ms = per_call_ms(calls32)
     i32, c32 = layer32.idx.cpu().numpy(), layer32.counts.cpu().numpy()
     f32 = sparse_flops(i32, c32, wl32.n_heads, wl32.head_dim, wl32.block)
     tiles32 = 0
@@ -601,18 +591,13 @@ def main():
         O_o = torch.empty_like(st_o[0][0])
         for t in range(wo.n_discovery + 1):
             lay_o.step(t, *st_o[t], O_o)
-        ev_o = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(2 * n_t)]
-        for rep in range(2):  # the first pass warms up
-            for i, t in enumerate(range(wo.n_discovery, wo.n_discovery + n_t)):
-                ev_o[i][0].record(stream)
-                wise.wise_sparse_attn(sh_o, *st_o[t], lay_o.idx, lay_o.counts, O_o)
-                ev_o[i][1].record(stream)
-                ev_o[n_t + i][0].record(stream)
-                wise.wise_full_attn_accumulate(sh_o, *st_o[t], O_o)
-                ev_o[n_t + i][1].record(stream)
-            torch.cuda.synchronize()
-        sp = statistics.mean(a.elapsed_time(b) for a, b in ev_o[:n_t])
-        dn = statistics.mean(a.elapsed_time(b) for a, b in ev_o[n_t:])
+        sp_calls = [lambda t=t: wise.wise_sparse_attn(sh_o, *st_o[t], lay_o.idx, lay_o.counts, O_o)
+                    for t in range(wo.n_discovery, wo.n_discovery + n_t)]
+        dn_calls = [lambda t=t: wise.wise_full_attn_accumulate(sh_o, *st_o[t], O_o)
+                    for t in range(wo.n_discovery, wo.n_discovery + n_t)]
+        per_call_ms(sp_calls + dn_calls)  # warm-up
+        sp = per_call_ms(sp_calls)
+        dn = per_call_ms(dn_calls)
         f_o = sparse_flops(lay_o.idx.cpu().numpy(), lay_o.counts.cpu().numpy(), wo.n_heads, wo.head_dim, wo.block)
         other[name] = {"late_ms": round(sp, 5), "dense_ms": round(dn, 5), "speedup_vs_dense": round(dn / sp, 4),
                        "tflops_effective": round(f_o / (sp * 1e-3) / 1e12, 2),

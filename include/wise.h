@@ -28,6 +28,12 @@
  *    out) are recorded in a per-device status word read by wise_get_status().
  *  - Empty problems (batch == 0 or seqlen == 0) return WISE_OK and launch
  *    nothing.
+ *  - The attention calls (wise_full_attn_accumulate and its _noalloc variant,
+ *    wise_sparse_attn, wise_freeze_a_attn) are launched as programmatic
+ *    dependents: their set-up, and their reads of idx and counts, may overlap
+ *    the end of the preceding attention call on the same stream, whose other
+ *    effects they wait for.  So idx and counts must not share memory with the
+ *    O or blockmass of the preceding attention call.
  *  - Inputs are never written.  The library keeps one lazily allocated
  *    scratch buffer per device for the block-mass epilogue (see
  *    wise_full_attn_accumulate); no other call allocates device memory.

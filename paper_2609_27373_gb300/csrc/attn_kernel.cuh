@@ -370,6 +370,8 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
       }
       ++jt;
       if (first) {
+        // The first copy: the previous kernel of the stream has completed.
+        if (nq == 0) griddep_wait();
         // The staging buffer is free once the previous unit's Q is in TMEM.
         if (nq >= 1 && !mbar_wait(&sb.q_stage_free, (nq - 1) & 1, abort, p.wait_ns)) {
           ok = false;
@@ -415,6 +417,7 @@ __device__ void attn_producer(const CUtensorMap* mapQ, const CUtensorMap* mapK, 
   if (ok) mbar_arrive(&sb.k_full[jk % RK]);
   if (ok && jv >= RV && !mbar_wait(&sb.v_empty[jv % RV], ((jv / RV) - 1) & 1, abort, p.wait_ns)) ok = false;
   if (ok) mbar_arrive(&sb.v_full[jv % RV]);
+  if (nq == 0) griddep_wait();  // no copy was issued; the status word is written after the wait
   if (bad) atomicOr(p.status, kStatusBadSupport);
   if (!ok) {
     raise_status(p, &sb.abort, kStatusTimeout);
@@ -939,6 +942,16 @@ __global__ void __launch_bounds__(AttnCfg<D>::kThreads, 1)
   __syncthreads();
   tc_fence_after_sync();
   const uint32_t tmem = sb.tmem_base;
+  // Set-up above touched no global memory: with a programmatic launch it
+  // overlaps the tail of the previous kernel of the stream.  Every access to
+  // Q, K, V, O and blockmass comes after the wait; the producer and the
+  // schedule stager may read idx and counts before it (the only kernels
+  // that launch this one early are attention kernels, which write O and
+  // blockmass only), so the producer waits just before its first copy.  The
+  // next kernel may then be scheduled; its CTAs take SMs as this grid's CTAs
+  // exit.
+  if (warp != C::kProducerWarp && warp != 11) griddep_wait();
+  if (threadIdx.x == 0) griddep_launch_dependents();
 
   if (warp < 8) {
     warpgroup_reg_inc<C::kRegsSoftmax>();
@@ -972,7 +985,20 @@ cudaError_t launch_attn_instance(const AttnLaunch& L) {
   auto kern = attn_kernel<D, BLK, MODE>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemLaunch);
   if (e != cudaSuccess) return e;
-  kern<<<L.grid, C::kThreads, C::kSmemLaunch, L.stream>>>(L.mapQ, L.mapK, L.mapV, L.mapO, L.p);
+  // Programmatic stream serialization: the grid may be scheduled while the
+  // previous kernel of the stream finishes (see griddep_wait in the kernel).
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(L.grid);
+  cfg.blockDim = dim3(C::kThreads);
+  cfg.dynamicSmemBytes = C::kSmemLaunch;
+  cfg.stream = L.stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, kern, L.mapQ, L.mapK, L.mapV, L.mapO, L.p);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

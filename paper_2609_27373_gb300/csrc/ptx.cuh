@@ -257,6 +257,17 @@ __device__ __forceinline__ void umma_ts_split(uint32_t d_tmem, uint32_t a_tmem, 
       : "memory");
 }
 
+// Programmatic dependent launch.  griddep_wait: returns once every grid this
+// one depends on in its stream has completed and its memory operations are
+// visible (immediately when the kernel was not launched as a dependent).
+// griddep_launch_dependents: this CTA lets the next kernel of the stream be
+// scheduled before this grid completes (its CTAs still wait in griddep_wait
+// before touching memory).
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // Arrive once on `bar` when every tcgen05.mma issued so far by this thread
 // has completed.
 __device__ __forceinline__ void umma_commit(uint64_t* bar) {
