@@ -94,11 +94,15 @@ struct AttnCfg {
   // Epilogue staging: per softmax warp of L, 32 rows x 64 columns of O
   // (one 128-byte-swizzled TMA box).
   static constexpr int kOutBytes = 4 * 32 * 128;
-  static constexpr int kRingFit = (kBudget - kQBytes - kOutBytes) / kKVBytes;
+  // Block-mass epilogue: per-warp column sums [2 buffers][4 warps][key
+  // blocks] for up to kMassWsBlocks key blocks (more go to the global scratch).
+  static constexpr int kMassWsBlocks = 128;
+  static constexpr int kMassWsBytes = 2 * 4 * kMassWsBlocks * 4;
+  static constexpr int kRingFit = (kBudget - kQBytes - kOutBytes - kMassWsBytes) / kKVBytes;
   static constexpr int kRing = kRingFit > 12 ? 12 : kRingFit;
   static constexpr int kRingK = (kRing + 1) / 2;  // K tiles (consumed by S)
   static constexpr int kRingV = kRing / 2;        // V tiles (consumed by P V)
-  static constexpr int kSmemBytes = kQBytes + kRing * kKVBytes + kOutBytes + 1024;
+  static constexpr int kSmemBytes = kQBytes + kRing * kKVBytes + kOutBytes + kMassWsBytes + 1024;
   // At least 116 KB so that a single CTA resides per SM (it owns all 512
   // TMEM columns).
   static constexpr int kSmemLaunch = kSmemBytes > 116 * 1024 ? kSmemBytes : 116 * 1024;
@@ -561,6 +565,7 @@ struct EpiInfo {
 // ------------------------------------------------------------------- softmax
 template <int D, int BLK, int MODE>
 __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w, uint32_t tmem, uint8_t* out_stage,
+                             float* mass_ws,
                              SharedState<AttnCfg<D>::kRingK, AttnCfg<D>::kRingV>& sb) {
   using C = AttnCfg<D>;
   constexpr float kRescaleThreshold = 8.0f;   // log2 units: P stays <= 256
@@ -694,6 +699,42 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     // O refers to L's max, which is the final running max; E's is at most
     // that.
     const float l_row = (mE == -INFINITY) ? ei.l : ei.l + lE * ex2_approx(mE - ei.m);
+    int b, h, qt;
+    decode_unit(p, ei.u, b, h, qt);
+    const int row = qt * 128 + r;
+    // kDenseMass: the row's first 32 partial masses (E wrote its tiles'
+    // before publishing its part) and the block masses this epilogue adds to
+    // are loaded now, so that their latency overlaps the wait for the last
+    // P V and the output of O.  Dense variants: tile t of the unit is key
+    // tile t, holding key blocks t * S .. t * S + S - 1.
+    constexpr int kPrefetch = 2;  // block masses prefetched per thread
+    const int n_kb = min(ei.n_kt * S, p.n_blocks);
+    float v[32], prev[kPrefetch];
+    auto load_lc = [&](int kb0) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        const int kb = kb0 + i, t = kb / S;
+        v[i] = (kb < n_kb) ? *lc_at((ei.j0 + t) & 1, ei.nu, t, kb - t * S) : -INFINITY;
+      }
+    };
+    // Block mass entry e (= qi * n_blocks + kb) of this unit, or null when
+    // its query block lies past the end.
+    auto mass_at = [&](int e) -> float* {
+      const int qi = e / p.n_blocks, kb = e - qi * p.n_blocks;
+      const int qblock = qt * S + qi;
+      return qblock < p.n_blocks
+                 ? p.blockmass + ((size_t)(b * p.n_heads + h) * p.n_blocks + qblock) * p.n_blocks + kb
+                 : nullptr;
+    };
+    if constexpr (MODE == kDenseMass) {
+      load_lc(0);
+#pragma unroll
+      for (int i = 0; i < kPrefetch; ++i) {
+        const int e = r + 128 * i;
+        float* out = (p.step > 0 && e < S * p.n_blocks && e % p.n_blocks < n_kb) ? mass_at(e) : nullptr;
+        prev[i] = out ? *out : 0.0f;
+      }
+    }
     // P V(j1-2) completed before P(j1) was written, so o_full[j1 & 1] is at
     // most one phase short of P V(j1).
     if (!warp_wait(&sb.o_full[ei.j1 & 1], (ei.j1 >> 1) & 1, abort, p.wait_ns)) return false;
@@ -703,9 +744,6 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     tc_fence_before_sync();
     __syncwarp();
     if (lane == 0) mbar_arrive(&sb.o_free);
-    int b, h, qt;
-    decode_unit(p, ei.u, b, h, qt);
-    const int row = qt * 128 + r;
     const float inv_l = l_row > 0.0f ? 1.0f / l_row : 0.0f;
     // O / l through this warp's staging box (32 rows x 64 columns, 128-byte
     // swizzle): each thread writes its row, then the warp reads the box back
@@ -743,25 +781,24 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     }
     if constexpr (MODE == kDenseMass) {
       // Block mass (Eq. 5): per row 2^(lc - lse), summed over the rows of
-      // each query block.  E wrote its tiles' lc before publishing its part.
+      // each query block.
       const float lse = ei.m + lg2_approx(l_row);
-      float* ws = warp_sums + (size_t)(w * 2 + (n_epi & 1)) * 4 * p.n_blocks;
-      // Dense variants: tile t of the unit is key tile t, holding key blocks
-      // t * S .. t * S + S - 1.
-      const int n_kb = min(ei.n_kt * S, p.n_blocks);
+      // Per-warp column sums: in shared memory when the key blocks fit
+      // (double-buffered: a warp may start the next epilogue of its
+      // warpgroup while another still reads this one's), else in the global
+      // scratch.  The epilogues of the two warpgroups never overlap.
+      const bool ws_shared = p.n_blocks <= C::kMassWsBlocks;
+      const int ws_stride = ws_shared ? C::kMassWsBlocks : p.n_blocks;
+      float* ws = ws_shared ? mass_ws + (n_epi & 1) * 4 * C::kMassWsBlocks
+                            : warp_sums + (size_t)(w * 2 + (n_epi & 1)) * 4 * p.n_blocks;
       // 32 key blocks per pass: their partials are loaded together, and the
       // warp's 32 column sums end one per lane.
       for (int kb0 = 0; kb0 < n_kb; kb0 += 32) {
-        float v[32];
-#pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const int kb = kb0 + i, t = kb / S;
-          v[i] = (kb < n_kb) ? *lc_at((ei.j0 + t) & 1, ei.nu, t, kb - t * S) : -INFINITY;
-        }
+        if (kb0 > 0) load_lc(kb0);
 #pragma unroll
         for (int i = 0; i < 32; ++i) v[i] = (row < p.seqlen) ? ex2_approx(v[i] - lse) : 0.0f;
         const float sum = warp_column_sums(v, lane);
-        if (kb0 + lane < n_kb) ws[wq * p.n_blocks + kb0 + lane] = sum;
+        if (kb0 + lane < n_kb) ws[wq * ws_stride + kb0 + lane] = sum;
       }
       // Orders the four warps' writes before the reads below (release /
       // acquire at CTA scope).
@@ -770,17 +807,22 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
       if (!warp_wait(&sb.epi[w], n_epi & 1, abort, p.wait_ns)) return false;
       constexpr int kWarpsPerBlock = BLK / 32;  // warps holding one query block's rows
       const float inv_b = 1.0f / (float)BLK;
-      for (int e = r; e < S * p.n_blocks; e += 128) {
-        const int qi = e / p.n_blocks, kb = e % p.n_blocks;
-        const int qblock = qt * S + qi;
-        if (qblock >= p.n_blocks) continue;
-        float* out = p.blockmass + ((size_t)(b * p.n_heads + h) * p.n_blocks + qblock) * p.n_blocks + kb;
+      for (int i = 0, e = r; e < S * p.n_blocks; ++i, e += 128) {
+        const int qi = e / p.n_blocks, kb = e - qi * p.n_blocks;
+        float* out = mass_at(e);
+        if (!out) continue;
         if (kb < n_kb) {
           float sum = 0.0f;
 #pragma unroll
-          for (int q = qi * kWarpsPerBlock; q < (qi + 1) * kWarpsPerBlock; ++q) sum += ws[q * p.n_blocks + kb];
+          for (int q = qi * kWarpsPerBlock; q < (qi + 1) * kWarpsPerBlock; ++q) sum += ws[q * ws_stride + kb];
           sum *= inv_b;
-          *out = (p.step == 0) ? sum : *out + sum;
+          float before = 0.0f;
+          if (p.step > 0) {
+            before = i >= kPrefetch ? *out : prev[0];
+#pragma unroll
+            for (int k = 1; k < kPrefetch; ++k) before = (i == k) ? prev[k] : before;
+          }
+          *out = before + sum;
         } else if (p.step == 0) {
           *out = 0.0f;
         }
@@ -885,7 +927,8 @@ __global__ void __launch_bounds__(AttnCfg<D>::kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* q_stage = smem;             // one Q tile
   uint8_t* ring = smem + C::kQBytes;   // kRing K/V entries
-  uint8_t* out_stage = ring + C::kRing * C::kKVBytes;  // epilogue staging (1024-byte aligned)
+  uint8_t* out_stage = ring + C::kRing * C::kKVBytes;  // epilogue staging (1024-byte aligned), then the
+                                                       // block-mass column sums
   __shared__ SS sb;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -955,7 +998,8 @@ __global__ void __launch_bounds__(AttnCfg<D>::kThreads, 1)
 
   if (warp < 8) {
     warpgroup_reg_inc<C::kRegsSoftmax>();
-    attn_softmax<D, BLK, MODE>(&mapO, p, warp >> 2, tmem, out_stage, sb);
+    attn_softmax<D, BLK, MODE>(&mapO, p, warp >> 2, tmem, out_stage,
+                               reinterpret_cast<float*>(out_stage + C::kOutBytes), sb);
   } else {
     warpgroup_reg_dec<C::kRegsOther>();
     if (warp == C::kProducerWarp) {
