@@ -757,6 +757,7 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
     // epilogue of its own.
     uint8_t* stage = out_stage + wq * (32 * 128);
     __nv_bfloat16* o_rows = p.O + ((size_t)(b * p.n_heads + h) * p.seqlen + qt * 128 + wq * 32) * D;
+    const float2 inv_l2 = make_float2(inv_l, inv_l);  // O / l two columns per packed multiply
 #pragma unroll
     for (int hb = 0; hb < C::kBoxes; ++hb) {
 #pragma unroll
@@ -764,8 +765,13 @@ __device__ void attn_softmax(const CUtensorMap* mapO, const AttnParams& p, int w
         const int col = hb * 64 + c * 8;
         uint32_t q[4];
 #pragma unroll
-        for (int e = 0; e < 4; ++e)
-          q[e] = (col + 2 * e + 1 < D) ? pack_bf16x2(o[col + 2 * e] * inv_l, o[col + 2 * e + 1] * inv_l) : 0u;
+        for (int e = 0; e < 4; ++e) {
+          q[e] = 0u;
+          if (col + 2 * e + 1 < D) {
+            const float2 x = __fmul2_rn(make_float2(o[col + 2 * e], o[col + 2 * e + 1]), inv_l2);
+            q[e] = pack_bf16x2(x.x, x.y);
+          }
+        }
         st_shared_v4(smem_u32(stage + lane * 128 + ((c ^ (lane & 7)) << 4)), q[0], q[1], q[2], q[3]);
       }
       __syncwarp();
