@@ -390,6 +390,15 @@ def main():
                    for t in range(wl.n_discovery, wl.steps)]
     dense_ms = [per_call_ms(dense_calls) for _ in range(max(1, args.steps // 2))]
 
+    # ---- the discovery steps back to back, as they run in a trajectory (the
+    # per-step events above keep consecutive launches apart), timed like the
+    # dense baseline: as many launches (passes over the discovery steps' own
+    # inputs), into a scratch mass so that the layer's own stays as selected
+    disc_mass = torch.zeros_like(layer.blockmass)
+    disc_calls = [lambda t=t % wl.n_discovery: wise.wise_full_attn_accumulate(shape, *dev_steps[t], O, disc_mass, t)
+                  for t in range(len(dense_calls))]
+    disc_b2b_ms = [per_call_ms(disc_calls) for _ in range(max(1, args.steps // 2))]
+
     # ---- end to end through host buffers (pinned), late steps
     pinned = [tuple(torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).pin_memory() for x in host_steps[t])
               for t in range(wl.n_discovery, min(wl.steps, wl.n_discovery + 4))]
@@ -662,7 +671,8 @@ def main():
         "speedup_vs_dense": round(dense / rank_value, 4),
         "setup_inclusive_speedup": round(n_late * dense / (statistics.mean(sel_ms) + n_late * rank_value), 4),
         "trajectory_speedup": round(wl.steps * dense / step_ms, 4),
-        "discovery_ms": round(statistics.mean(disc_ms), 5),
+        "discovery_ms": round(statistics.mean(disc_b2b_ms), 5),
+        "discovery_event_ms": round(statistics.mean(disc_ms), 5),
         "select_ms": round(statistics.mean(sel_ms), 5),
         "tflops_effective": round(achieved, 2),
         "dense_tflops": round(flops_dense / (dense * 1e-3) / 1e12, 2),
