@@ -17,7 +17,8 @@ enum AttnMode : int { kDense = 0, kDenseMass = 1, kSparse = 2 };
 // masses [2 warpgroups][2 units][n_tiles / 2 + 1][sub][128 rows] (a
 // warpgroup handles every other tile of a unit, and keeps the previous unit's
 // values until its epilogue has read them), then per-warp column sums
-// [2 warpgroups][2][4 warps][n_blocks].
+// [2 warpgroups][2][4 warps][n_blocks] (used only when the kernel's shared
+// memory copy of them, for up to 128 key blocks, is too small).
 __host__ __device__ constexpr size_t scratch_floats_per_cta(int n_tiles, int sub, int n_blocks) {
   return (size_t)512 * sub * (n_tiles / 2 + 1) + (size_t)16 * n_blocks;
 }
