@@ -15,6 +15,10 @@ Reported (one JSON line on rank 0):
                    trajectory, divided by their number; mean over trajectories)
   dense_ms         the library's own dense kernel (no mass) on the same late
                    inputs, timed the same way; speedup = dense_ms / value
+  discovery_ms     the dense kernel with the block-mass epilogue on the
+                   discovery steps' inputs, timed the same way (as many
+                   launches as dense_ms); discovery_event_ms keeps the events
+                   around each discovery step of the timed trajectories
   roofline         the sparse kernel's algorithmic tensor FLOPs per launch
                    over its mean launch time, against the measured bf16 peak
   e2e              the same late step through the C ABI with Q/K/V copied from
